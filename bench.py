@@ -1,0 +1,489 @@
+#!/usr/bin/env python3
+"""Throughput of the four fused composite sparse expressions on GB300.
+
+One step = one pass of the whole hot path: the four fused expressions of the
+SparseLNR benchmark set (Sec. 6.2) at their full synthetic sizes,
+  <SDDMM,SpMM>  R-MAT 100k x 100k, 2M nnz, L = K = 64
+  <SpMM,GEMM>   R-MAT 2^20 x 2^20, 16.8M nnz, K = L = 128
+  MTTKRP        CSF 10k^3, 10M nnz, Zipf(1.2) slices, L = 32
+  <SpTTM,SpTTM> CSF 5k^3, 20M nnz, power-law fibers (mean 8), L = M = 64
+each through the C ABI with inputs resident in HBM.  L2 is flushed (a write of
+2x its size) before every expression, outside the timed events.  Metric:
+useful GFLOP/s (the flops the fused schedule must do, Sec. 3.1.3 / 6.2
+complexity) over the step; per-expression GFLOP/s, time and achieved HBM
+GB/s (minimum bytes / time) are reported beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl slnr|reference]
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+expressions need no exchange between GPUs); value = all ranks' flops / the
+slowest rank's time.  --impl reference times the CPU oracle instead (on rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+BENCH_CONFIGS = (1, 2, 3, 4)   # full-size workloads timed in one step (index 0 is the small parity case)
+
+
+# ---------------------------------------------------------------------------
+# algorithmic counts
+
+def _distinct(a) -> int:
+    if a.shape[0] == 0:
+        return 0
+    return int(np.unique(a).shape[0])
+
+
+def row_sizes(w):
+    """Work units of each expression's output rows and their nonzero counts."""
+    if w.op in ("spmm_gemm", "sddmm_spmm"):
+        return np.diff(w.B.pos).astype(np.int64)
+    if w.op == "spttm_ttm":
+        return np.diff(w.B.pos3).astype(np.int64)
+    sizes = np.zeros(w.B.dims[0], np.int64)
+    fib = np.diff(w.B.pos3).astype(np.int64)
+    if w.B.nfibers:
+        sizes[w.B.crd1] = np.add.reduceat(fib, w.B.pos2[:-1]) if w.B.nslices else 0
+    return sizes
+
+
+def row_flops(w) -> np.ndarray:
+    """Useful flops per output row under the fused schedule (Sec. 6.2 complexities)."""
+    d = w.dims
+    if w.op == "spmm_gemm":      # 2 nnz K + 2 K L per non-empty row
+        n = np.diff(w.B.pos).astype(np.int64)
+        return 2 * n * d["K"] + 2 * (n > 0) * d["K"] * d["L"]
+    if w.op == "sddmm_spmm":     # per nonzero: dot (2L), scale (1), axpy (2K)
+        n = np.diff(w.B.pos).astype(np.int64)
+        return n * (2 * d["L"] + 1 + 2 * d["K"])
+    if w.op == "mttkrp":         # 2 nnz L + 2 nfibers L, per slice
+        L = d["L"]
+        f = np.zeros(w.B.dims[0], np.int64)
+        if w.B.nslices:
+            fib_nnz = np.diff(w.B.pos3).astype(np.int64)
+            nnz_s = np.add.reduceat(fib_nnz, w.B.pos2[:-1]) if w.B.nfibers else np.zeros(w.B.nslices, np.int64)
+            nfib_s = np.diff(w.B.pos2).astype(np.int64)
+            f[w.B.crd1] = 2 * nnz_s * L + 2 * nfib_s * L
+        return f
+    if w.op == "spttm_ttm":      # 2 nnz L + 2 L M per fiber
+        n = np.diff(w.B.pos3).astype(np.int64)
+        return 2 * n * d["L"] + 2 * d["L"] * d["M"]
+    raise ValueError(w.op)
+
+
+def useful_flops(w) -> int:
+    return int(row_flops(w).sum())
+
+
+def min_bytes(w) -> int:
+    """Bytes an ideal evaluation moves: sparse structure and values once, each
+    dense operand row that is actually referenced once, every output once."""
+    d, B = w.dims, w.B
+    if w.op == "spmm_gemm":
+        K, L = d["K"], d["L"]
+        return 4 * (B.nrows + 1) + 8 * B.nnz + 4 * K * _distinct(B.crd) + 4 * K * L + 4 * B.nrows * L
+    if w.op == "sddmm_spmm":
+        K, L = d["K"], d["L"]
+        nonempty = int(np.count_nonzero(np.diff(B.pos)))
+        cols = _distinct(B.crd)
+        return 4 * (B.nrows + 1) + 8 * B.nnz + 4 * L * nonempty + 4 * (L + K) * cols + 4 * B.nrows * K
+    structure = 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers + 4 * (B.nfibers + 1) + 8 * B.nnz
+    if w.op == "mttkrp":
+        L = d["L"]
+        return structure + 4 * L * (_distinct(B.crd2) + _distinct(B.crd3)) + 4 * B.dims[0] * L
+    if w.op == "spttm_ttm":
+        L, M = d["L"], d["M"]
+        out_index = 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers
+        return structure + 4 * L * _distinct(B.crd3) + 4 * L * M + 4 * B.nfibers * M + out_index
+    raise ValueError(w.op)
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2205_11622_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            h.update(name.encode())
+            h.update(open(os.path.join(csrc, name), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        j = json.load(open(p))
+        return float(j["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def ncu_traffic(expr_name: str):
+    """DRAM bytes per call of an expression from the committed ncu summary, if it
+    was taken on the current kernel sources (else None)."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    if not os.path.exists(p):
+        return None
+    j = json.load(open(p))
+    if j.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    e = j.get("expressions", {}).get(expr_name)
+    return None if e is None else float(e["dram_bytes_per_call"])
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_uuid: str | None):
+        self.samples, self.proc, self.thread = [], None, None
+        self.uuid = gpu_uuid
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                self.samples.append(parts)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["clocks not sampled"]}
+        sm = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        mx = [float(s[2]) for s in self.samples if s[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for s in self.samples for n, v in zip(names, s[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a bounded sample (the cpu_baseline leg and the reference arm)
+
+def oracle_sample(w, flop_budget: float, seed: int):
+    """Seeded uniform sample of output rows whose useful flops reach flop_budget."""
+    rf = row_flops(w)
+    rng = np.random.default_rng(seed)
+    order = rng.permutation(rf.shape[0])
+    cum = np.cumsum(rf[order])
+    n = int(np.searchsorted(cum, flop_budget)) + 1
+    rows = np.sort(order[:max(1, min(n, order.shape[0]))]).astype(np.int32)
+    return rows, int(rf[rows].sum())
+
+
+def time_oracle(ws, flop_budget: float, seed: int = 11):
+    import oracle
+    orc = oracle.get()
+    secs, flops, parts = 0.0, 0, []
+    for w in ws:
+        rows, f = oracle_sample(w, flop_budget, seed)
+        t0 = time.perf_counter()
+        orc.run(w, rows=rows)
+        dt = time.perf_counter() - t0
+        secs += dt
+        flops += f
+        parts.append(f"{w.name}: {rows.shape[0]} rows, {f / 1e9:.2f} GFLOP, {dt:.2f} s")
+    return flops, secs, "; ".join(parts)
+
+
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    ws = [wl.full(i) for i in BENCH_CONFIGS]
+    budget = args.ref_gflop_per_expr * 1e9
+    times, flops_total, sample = [], 0, ""
+    for step in range(args.warmup + args.steps):
+        flops, secs, sample = time_oracle(ws, budget, seed=100 + step)
+        if step >= args.warmup:
+            times.append(secs)
+            flops_total += flops
+    secs = sum(times)
+    value = flops_total / secs / 1e9
+    line = {
+        "impl": "reference", "metric": "useful GFLOP/s (4 fused sparse expressions)", "value": round(value, 4),
+        "unit": "GFLOP/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * secs / args.steps, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_block(ws),
+        "cpu_baseline": {"value": round(value, 4), "unit": "GFLOP/s", "cores": 1, "kind": "oracle",
+                         "sample": "per step, a seeded uniform sample of output rows of each expression worth "
+                                   f"{args.ref_gflop_per_expr} GFLOP (oracle computes value and magnitude "
+                                   f"companion in fp64, single thread); last step: {sample}"},
+        "e2e": {"value": round(value, 4), "unit": "GFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def config_block(ws):
+    return {
+        "workload": " + ".join(w.name for w in ws),
+        "expressions": {w.name: w.recipe for w in ws},
+        "l2": "flushed before every expression by writing a buffer of 2x the L2 size (outside the timed events)",
+        "variant": "fused", "allow_tf32": True,
+        "parallelism": "replicas (one independent full step per GPU)",
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["slnr", "reference"], default="slnr")
+    ap.add_argument("--variant", choices=["fused", "unfused"], default="fused")
+    ap.add_argument("--no-tf32", action="store_true")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--cpu-gflop-per-expr", type=float, default=4.0)
+    ap.add_argument("--ref-gflop-per-expr", type=float, default=1.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import torch
+
+    import paper_2205_11622_gb300 as slnr
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    slnr.build()
+    slnr.lib()
+    allow_tf32 = not args.no_tf32
+
+    ws = [wl.full(i) for i in BENCH_CONFIGS]
+    flops = [useful_flops(w) for w in ws]
+    mbytes = [min_bytes(w) for w in ws]
+
+    # device-resident inputs, preallocated outputs and workspaces
+    def upload(w):
+        if w.op in ("spmm_gemm", "sddmm_spmm"):
+            B = slnr.DeviceCSR.from_host(w.B, dev)
+        else:
+            B = slnr.DeviceCSF3.from_host(w.B, dev)
+        dense = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev) for k, v in w.dense.items()}
+        return B, dense
+
+    dev_inputs = [upload(w) for w in ws]
+    wspaces = [slnr.Workspace(device=dev) for _ in ws]
+    outs = [None] * len(ws)
+
+    def call(i, out=None):
+        w = ws[i]
+        B, dense = dev_inputs[i]
+        return slnr.run(w.op, B, dense, out=out, variant=args.variant, allow_tf32=allow_tf32, workspace=wspaces[i])
+
+    for i in range(len(ws)):
+        outs[i] = call(i)
+    torch.cuda.synchronize()
+
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush_buf = torch.empty(max(2 * l2, 64 << 20), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    slnr.timing_enable(True)
+
+    def one_step(record):
+        per_expr, per_kernel, launches = [], [], 0
+        for i in range(len(ws)):
+            flush_buf.fill_(i & 0xFF)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            call(i, out=outs[i])
+            b.record(stream)
+            b.synchronize()
+            per_expr.append(a.elapsed_time(b))
+            kt = slnr.timing_read()
+            per_kernel.append(kt)
+            launches += len(kt)
+        return per_expr, per_kernel, launches
+
+    for _ in range(args.warmup):
+        one_step(False)
+    torch.cuda.synchronize()
+    if pg is not None:
+        pg.barrier()
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        uuid = None
+    clocks = ClockSampler(uuid)
+    clocks.start()
+    time.sleep(0.5)
+    torch.cuda.synchronize()
+    expr_ms = [[] for _ in ws]
+    kern_ms = [dict() for _ in ws]
+    gpu_launches = 0
+    for _ in range(args.steps):
+        pe, pk, nl = one_step(True)
+        gpu_launches += nl
+        for i in range(len(ws)):
+            expr_ms[i].append(pe[i])
+            for name, ms in pk[i]:
+                kern_ms[i][name] = kern_ms[i].get(name, 0.0) + ms
+    torch.cuda.synchronize()
+    time.sleep(0.3)
+    clocks.stop()
+    mean_ms = [statistics.mean(x) for x in expr_ms]
+    step_ms = sum(mean_ms)
+    if pg is not None:
+        t = torch.tensor([step_ms], dtype=torch.float64, device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        step_ms = float(t.item())
+        pg.barrier()
+    total_flops = sum(flops)
+    value = world * total_flops / (step_ms / 1e3) / 1e9
+
+    peak, peak_kind = measured_peaks()
+    per_expression = {}
+    for i, w in enumerate(ws):
+        kms = {k: round(v / args.steps, 4) for k, v in kern_ms[i].items()}
+        per_expression[w.name] = {
+            "ms": round(mean_ms[i], 4), "gflops": round(flops[i] / (mean_ms[i] / 1e3) / 1e9, 2),
+            "min_bytes": mbytes[i], "gbs": round(mbytes[i] / (mean_ms[i] / 1e3) / 1e9, 1),
+            "hbm_frac": round(mbytes[i] / (mean_ms[i] / 1e3) / 1e9 / peak, 4),
+            "kernels_ms": kms, "useful_flops": flops[i]}
+    dom = int(np.argmax(mean_ms))
+    dw = ws[dom]
+    achieved = mbytes[dom] / (mean_ms[dom] / 1e3) / 1e9
+    traffic = ncu_traffic(dw.name)
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": traffic,
+                "kernel": f"{dw.name}: the fused call (launches {', '.join(kern_ms[dom].keys())}), "
+                          f"{mbytes[dom]} algorithmic bytes per call",
+                "peak_kind": f"{peak_kind} HBM copy bandwidth"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        cf, cs, sample = time_oracle(ws, args.cpu_gflop_per_expr * 1e9)
+        cpu = {"value": round(cf / cs / 1e9, 4), "unit": "GFLOP/s", "cores": 1, "kind": "oracle",
+               "sample": f"seeded uniform sample of output rows per expression (oracle computes value and "
+                         f"magnitude companion in fp64, single thread): {sample}"}
+
+    e2e = None
+    if not args.skip_e2e:
+        e2e = measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, args.steps, total_flops, world, pg, dev)
+
+    line = {
+        "metric": "useful GFLOP/s (4 fused sparse expressions)", "value": round(value, 2), "unit": "GFLOP/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32 (tf32 tensor-core contractions allowed)" if allow_tf32 else "f32",
+        "data": "synthetic", "config": config_block(ws), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": gpu_launches, "clocks": clocks.summary(), "per_expression": per_expression,
+    }
+    line["config"]["variant"] = args.variant
+    line["config"]["allow_tf32"] = allow_tf32
+    if rank == 0:
+        print(json.dumps(line))
+    if pg is not None:
+        pg.destroy_process_group()
+    return 0
+
+
+def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_flops, world, pg, dev):
+    """Same step through the public API with host buffers: every step copies all
+    inputs from pinned host memory to the device and all outputs back."""
+    host_in, dev_in, host_out, dev_out = [], [], [], []
+    for i, w in enumerate(ws):
+        B, dense = dev_inputs[i]
+        arrays = [getattr(B, f) for f in ("pos", "crd", "vals")] if w.op in ("spmm_gemm", "sddmm_spmm") else \
+            [getattr(B, f) for f in ("pos1", "crd1", "pos2", "crd2", "pos3", "crd3", "vals")]
+        arrays += list(dense.values())
+        for a in arrays:
+            dev_in.append(a)
+            host_in.append(a.cpu().pin_memory())
+        o = outs[i]
+        for t in (o if isinstance(o, tuple) else (o,)):
+            dev_out.append(t)
+            host_out.append(torch.empty(t.shape, dtype=t.dtype, pin_memory=True))
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+
+    def step():
+        for d, h in zip(dev_in, host_in):
+            d.copy_(h, non_blocking=True)
+        for i in range(len(ws)):
+            call(i, out=outs[i])
+        for h, d in zip(host_out, dev_out):
+            h.copy_(d, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    if pg is not None:
+        pg.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        step()
+    b.record(stream)
+    b.synchronize()
+    ms = a.elapsed_time(b) / steps
+    if pg is not None:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": round(world * total_flops / (ms / 1e3) / 1e9, 2), "unit": "GFLOP/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 3)}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

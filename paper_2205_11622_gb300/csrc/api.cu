@@ -1,0 +1,486 @@
+// C entry points of libslnr (declared in include/slnr.h): argument checks,
+// workspace layout, and the launch sequence of each variant.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "launch.h"
+
+using namespace slnr;
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+slnr_status fail(slnr_status st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+// ---------------------------------------------------------------------------
+// per-launch timing (slnr_timing_*): events recorded between launches
+
+constexpr int kMaxTimed = 16;
+struct Timing {
+  bool on = false;
+  bool created = false;
+  int n = 0;
+  const char* names[kMaxTimed] = {};
+  cudaEvent_t ev[kMaxTimed + 1] = {};
+};
+thread_local Timing g_timing;
+
+void timing_begin() { g_timing.n = 0; }
+
+void timing_mark(const char* name, cudaStream_t s) {
+  if (!g_timing.on || g_timing.n >= kMaxTimed) return;
+  cudaEventRecord(g_timing.ev[g_timing.n], s);
+  g_timing.names[g_timing.n++] = name;
+}
+
+void timing_end(cudaStream_t s) {
+  if (g_timing.on && g_timing.n > 0) cudaEventRecord(g_timing.ev[g_timing.n], s);
+}
+
+#define SLNR_CUDA(expr)                                                                   \
+  do {                                                                                    \
+    cudaError_t e_ = (expr);                                                              \
+    if (e_ != cudaSuccess) return fail(SLNR_ERR_CUDA, "%s: %s", #expr, cudaGetErrorString(e_)); \
+  } while (0)
+
+bool pow2_dim(int32_t d) { return d >= 4 && d <= 256 && (d & (d - 1)) == 0; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// ---------------------------------------------------------------------------
+// workspace layout (identical for the size query and the call)
+
+struct Layout {
+  size_t cur = sizeof(WsHeader);
+  size_t take(size_t bytes) {
+    cur = align256(cur);
+    const size_t o = cur;
+    cur += bytes;
+    return o;
+  }
+  // heavy-row split of a CSR-shaped level
+  size_t o_heavy = 0, o_chunks = 0, o_partial = 0;
+  int max_heavy = 0, max_chunks = 0;
+  void split(int64_t nrows, int64_t nnz, int width) {
+    if (nnz > kLightMax) {
+      int64_t mh = nnz / (kLightMax + 1);
+      if (mh > nrows) mh = nrows;
+      max_heavy = (int)mh;
+      max_chunks = (int)(nnz / kChunk + mh + 1);
+    }
+    o_heavy = take(sizeof(HeavyRow) * (size_t)max_heavy);
+    o_chunks = take(sizeof(Chunk) * (size_t)max_chunks);
+    o_partial = take(sizeof(float) * (size_t)max_chunks * (size_t)width);
+  }
+  // MTTKRP units
+  size_t o_su = 0, o_units = 0, o_upartial = 0;
+  int max_units = 0;
+  void units(int64_t nslices, int64_t nnz, int width) {
+    max_units = (int)(nnz / kUnitNnz + nslices + 1);
+    o_su = take(sizeof(SliceUnits) * (size_t)nslices);
+    o_units = take(sizeof(Unit) * (size_t)max_units);
+    o_upartial = take(sizeof(float) * (size_t)max_units * (size_t)width);
+  }
+  size_t o_inter = 0;
+  void inter(size_t bytes) { o_inter = take(bytes); }
+  size_t total() const { return align256(cur); }
+};
+
+SplitPlan split_plan(char* ws, const Layout& l) {
+  return SplitPlan{reinterpret_cast<WsHeader*>(ws), reinterpret_cast<HeavyRow*>(ws + l.o_heavy),
+                   reinterpret_cast<Chunk*>(ws + l.o_chunks), reinterpret_cast<float*>(ws + l.o_partial),
+                   l.max_heavy, l.max_chunks};
+}
+
+UnitPlan unit_plan(char* ws, const Layout& l) {
+  return UnitPlan{reinterpret_cast<WsHeader*>(ws), reinterpret_cast<SliceUnits*>(ws + l.o_su),
+                  reinterpret_cast<Unit*>(ws + l.o_units), reinterpret_cast<float*>(ws + l.o_upartial),
+                  l.max_units};
+}
+
+// ---------------------------------------------------------------------------
+// argument checks
+
+slnr_status check_opts(const slnr_opts* o) {
+  if (!o) return fail(SLNR_ERR_NULL, "opts is NULL");
+  if (o->variant != SLNR_FUSED && o->variant != SLNR_UNFUSED)
+    return fail(SLNR_ERR_UNSUPPORTED, "unknown variant %d", (int)o->variant);
+  if (o->reserved != 0) return fail(SLNR_ERR_UNSUPPORTED, "opts.reserved must be 0");
+  return SLNR_OK;
+}
+
+slnr_status check_csr(const slnr_csr* B, bool need_ptrs) {
+  if (!B) return fail(SLNR_ERR_NULL, "B is NULL");
+  if (B->nrows < 0 || B->ncols < 0 || B->nnz < 0) return fail(SLNR_ERR_SHAPE, "negative size in B");
+  if (B->nnz >= (int64_t(1) << 31)) return fail(SLNR_ERR_UNSUPPORTED, "nnz must be < 2^31");
+  if (B->nnz > 0 && (B->nrows == 0 || B->ncols == 0)) return fail(SLNR_ERR_SHAPE, "nnz > 0 in an empty matrix");
+  if (need_ptrs) {
+    if (!B->pos) return fail(SLNR_ERR_NULL, "B.pos is NULL");
+    if (B->nnz > 0 && (!B->crd || !B->vals)) return fail(SLNR_ERR_NULL, "B.crd or B.vals is NULL");
+  }
+  return SLNR_OK;
+}
+
+slnr_status check_csf(const slnr_csf3* B, bool need_ptrs) {
+  if (!B) return fail(SLNR_ERR_NULL, "B is NULL");
+  if (B->dim[0] < 0 || B->dim[1] < 0 || B->dim[2] < 0 || B->nnz < 0 || B->nslices < 0 || B->nfibers < 0)
+    return fail(SLNR_ERR_SHAPE, "negative size in B");
+  if (B->nnz >= (int64_t(1) << 31)) return fail(SLNR_ERR_UNSUPPORTED, "nnz must be < 2^31");
+  if (B->nslices > B->dim[0] || (int64_t)B->nfibers > (int64_t)B->nslices * B->dim[1] ||
+      B->nnz > (int64_t)B->nfibers * B->dim[2])
+    return fail(SLNR_ERR_SHAPE, "counts of B exceed its dimensions");
+  if (need_ptrs) {
+    if (!B->pos1 || !B->pos2 || !B->pos3) return fail(SLNR_ERR_NULL, "a CSF position array is NULL");
+    if (B->nslices > 0 && !B->crd1) return fail(SLNR_ERR_NULL, "B.crd1 is NULL");
+    if (B->nfibers > 0 && !B->crd2) return fail(SLNR_ERR_NULL, "B.crd2 is NULL");
+    if (B->nnz > 0 && (!B->crd3 || !B->vals)) return fail(SLNR_ERR_NULL, "B.crd3 or B.vals is NULL");
+  }
+  return SLNR_OK;
+}
+
+slnr_status check_dims(const char* what, int32_t d) {
+  if (d <= 0) return fail(SLNR_ERR_SHAPE, "%s = %d must be positive", what, (int)d);
+  if (!pow2_dim(d)) return fail(SLNR_ERR_UNSUPPORTED, "%s = %d: must be a power of two in [4, 256]", what, (int)d);
+  return SLNR_OK;
+}
+
+slnr_status check_dense(const char* what, const void* p) {
+  if (!p) return fail(SLNR_ERR_NULL, "%s is NULL", what);
+  if (!aligned16(p)) return fail(SLNR_ERR_UNSUPPORTED, "%s must be 16-byte aligned", what);
+  return SLNR_OK;
+}
+
+slnr_status check_ws(const slnr_opts* o, size_t need) {
+  if (!o->workspace) return fail(SLNR_ERR_WORKSPACE, "workspace is NULL (needs %zu bytes)", need);
+  if ((reinterpret_cast<uintptr_t>(o->workspace) & 255u) != 0)
+    return fail(SLNR_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (o->workspace_bytes < need)
+    return fail(SLNR_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", o->workspace_bytes, need);
+  return SLNR_OK;
+}
+
+// A kernel launch of the call: timing mark, then the launch, then its status.
+#define SLNR_LAUNCH(name, expr) \
+  do {                          \
+    timing_mark(name, s);       \
+    SLNR_CUDA(expr);            \
+  } while (0)
+
+#define SLNR_CHECK(expr)            \
+  do {                              \
+    slnr_status st_ = (expr);       \
+    if (st_ != SLNR_OK) return st_; \
+  } while (0)
+
+// Zero the header, then (validate mode) run the device check and wait for it.
+template <typename Launch>
+slnr_status begin(char* ws, cudaStream_t s, bool validate, Launch launch_validate) {
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(ws);
+  SLNR_CUDA(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), s));
+  if (validate) {
+    SLNR_CUDA(launch_validate(hdr));
+    int flag = 0;
+    SLNR_CUDA(cudaMemcpyAsync(&flag, &hdr->error, sizeof(int), cudaMemcpyDeviceToHost, s));
+    SLNR_CUDA(cudaStreamSynchronize(s));
+    if (flag != 0) return fail(SLNR_ERR_INDEX, "malformed index arrays (flags 0x%x)", flag);
+  }
+  return SLNR_OK;
+}
+
+// ---------------------------------------------------------------------------
+// layouts per operation
+
+Layout layout_spmm_gemm(const slnr_csr* B, int32_t K, int32_t L, int variant) {
+  (void)L;
+  Layout l;
+  l.split(B->nrows, B->nnz, K);
+  if (variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nrows * (size_t)K);
+  return l;
+}
+
+Layout layout_sddmm_spmm(const slnr_csr* B, int32_t L, int32_t K, int variant) {
+  (void)L;
+  Layout l;
+  l.split(B->nrows, B->nnz, K);
+  if (variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nnz);
+  return l;
+}
+
+Layout layout_mttkrp(const slnr_csf3* B, int32_t L, int variant) {
+  Layout l;
+  l.units(B->nslices, B->nnz, L);
+  if (variant == SLNR_UNFUSED) {
+    l.split(B->nfibers, B->nnz, L);
+    l.inter(sizeof(float) * (size_t)B->nfibers * (size_t)L);
+  }
+  return l;
+}
+
+Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, int variant) {
+  (void)M;
+  Layout l;
+  l.split(B->nfibers, B->nnz, L);
+  if (variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nfibers * (size_t)L);
+  return l;
+}
+
+CsrView csr_view(const slnr_csr* B) { return CsrView{B->nrows, B->ncols, B->nnz, B->pos, B->crd, B->vals}; }
+CsrView fiber_view(const slnr_csf3* B) {
+  return CsrView{B->nfibers, B->dim[2], B->nnz, B->pos3, B->crd3, B->vals};
+}
+
+}  // namespace
+
+// ===========================================================================
+
+extern "C" {
+
+const char* slnr_status_string(slnr_status s) {
+  switch (s) {
+    case SLNR_OK: return "SLNR_OK";
+    case SLNR_ERR_NULL: return "SLNR_ERR_NULL";
+    case SLNR_ERR_SHAPE: return "SLNR_ERR_SHAPE";
+    case SLNR_ERR_INDEX: return "SLNR_ERR_INDEX";
+    case SLNR_ERR_WORKSPACE: return "SLNR_ERR_WORKSPACE";
+    case SLNR_ERR_UNSUPPORTED: return "SLNR_ERR_UNSUPPORTED";
+    case SLNR_ERR_CUDA: return "SLNR_ERR_CUDA";
+    case SLNR_ERR_TIMEOUT: return "SLNR_ERR_TIMEOUT";
+  }
+  return "SLNR_ERR_UNKNOWN";
+}
+
+const char* slnr_last_error(void) { return g_last_error; }
+
+const char* slnr_version(void) { return "slnr 0.1.0 (sm_103a)"; }
+
+slnr_status slnr_timing_enable(int32_t on) {
+  if (on && !g_timing.created) {
+    for (int i = 0; i <= kMaxTimed; ++i) SLNR_CUDA(cudaEventCreate(&g_timing.ev[i]));
+    g_timing.created = true;
+  }
+  g_timing.on = on != 0;
+  g_timing.n = 0;
+  return SLNR_OK;
+}
+
+int32_t slnr_timing_count(void) { return g_timing.on ? g_timing.n : 0; }
+
+slnr_status slnr_timing_get(int32_t i, const char** name, float* ms) {
+  if (!g_timing.on || i < 0 || i >= g_timing.n) return fail(SLNR_ERR_SHAPE, "no timed launch %d", (int)i);
+  if (!name || !ms) return fail(SLNR_ERR_NULL, "name or ms is NULL");
+  SLNR_CUDA(cudaEventSynchronize(g_timing.ev[g_timing.n]));
+  SLNR_CUDA(cudaEventElapsedTime(ms, g_timing.ev[i], g_timing.ev[i + 1]));
+  *name = g_timing.names[i];
+  return SLNR_OK;
+}
+
+slnr_status slnr_spmm_gemm_workspace(const slnr_csr* B, int32_t K, int32_t L, const slnr_opts* opts,
+                                     size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, false));
+  SLNR_CHECK(check_dims("K", K));
+  SLNR_CHECK(check_dims("L", L));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_spmm_gemm(B, K, L, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_sddmm_spmm_workspace(const slnr_csr* B, int32_t L, int32_t K, const slnr_opts* opts,
+                                      size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, false));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("K", K));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_sddmm_spmm(B, L, K, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_mttkrp_workspace(const slnr_csf3* B, int32_t L, const slnr_opts* opts, size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, false));
+  SLNR_CHECK(check_dims("L", L));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_mttkrp(B, L, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_spttm_ttm_workspace(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opts* opts,
+                                     size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, false));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_spttm_ttm(B, L, M, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const float* D, int32_t L, float* A,
+                           const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, true));
+  SLNR_CHECK(check_dims("K", K));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_spmm_gemm(B, K, L, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->nrows == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
+  const CsrView v = csr_view(B);
+  const SplitPlan sp = split_plan(ws, l);
+  const int tf32 = opts->allow_tf32 != 0;
+  SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+  SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(K, v, C, sp, s));
+  if (opts->variant == SLNR_FUSED) {
+    SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(K, L, v, C, D, A, tf32, s));
+    SLNR_LAUNCH("combine", launch_combine(K, sp, D, L, A, s));
+  } else {
+    float* T = reinterpret_cast<float*>(ws + l.o_inter);
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(K, v, C, T, s));
+    SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, T, s));
+    SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, K, L, T, D, A, tf32, s));
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_sddmm_spmm(const slnr_csr* B, const float* C, const float* D, int32_t L, const float* E,
+                            int32_t K, float* A, const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, true));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("K", K));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("E", E));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_sddmm_spmm(B, L, K, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->nrows == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
+  const CsrView v = csr_view(B);
+  const SplitPlan sp = split_plan(ws, l);
+  SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+  if (opts->variant == SLNR_FUSED) {
+    SLNR_LAUNCH("sddmm_spmm_chunks", launch_sddmm_spmm_chunks(v, C, D, L, E, K, sp, s));
+    SLNR_LAUNCH("sddmm_spmm_rows", launch_sddmm_spmm_rows(v, C, D, L, E, K, A, s));
+    SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, A, s));
+  } else {
+    float* Y = reinterpret_cast<float*>(ws + l.o_inter);
+    SLNR_LAUNCH("sddmm_rows", launch_sddmm_rows(v, C, D, L, Y, s));
+    SLNR_LAUNCH("sddmm_chunks", launch_sddmm_chunks(v, C, D, L, Y, sp, s));
+    CsrView vy = v;
+    vy.vals = Y;
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(K, vy, E, sp, s));
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(K, vy, E, A, s));
+    SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, A, s));
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_mttkrp(const slnr_csf3* B, const float* C, const float* D, int32_t L, float* A,
+                        const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, true));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_mttkrp(B, L, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->dim[0] == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
+  const UnitPlan up = unit_plan(ws, l);
+  SLNR_LAUNCH("csf_units", launch_csf_units(*B, up, s));
+  if (opts->variant == SLNR_FUSED) {
+    SLNR_LAUNCH("mttkrp_units", launch_mttkrp_units(L, *B, C, D, up, s));
+  } else {
+    const CsrView fv = fiber_view(B);
+    const SplitPlan sp = split_plan(ws, l);
+    float* T = reinterpret_cast<float*>(ws + l.o_inter);
+    SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, fv, D, sp, s));
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, fv, D, T, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
+    SLNR_LAUNCH("mttkrp_stage2_units", launch_mttkrp_stage2_units(L, *B, T, C, up, s));
+  }
+  SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, A, s));
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const float* D, int32_t M,
+                           int32_t* A_pos1, int32_t* A_crd1, int32_t* A_pos2, int32_t* A_crd2, float* A_vals,
+                           const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, true));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  if (!A_pos1 || !A_pos2 || (B->nslices > 0 && !A_crd1) || (B->nfibers > 0 && !A_crd2))
+    return fail(SLNR_ERR_NULL, "an output index array of A is NULL");
+  if (B->nfibers > 0) SLNR_CHECK(check_dense("A_vals", A_vals));
+  const Layout l = layout_spttm_ttm(B, L, M, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
+  // A's two compressed levels are B's (the (i,j) pattern is unchanged)
+  SLNR_CUDA(cudaMemcpyAsync(A_pos1, B->pos1, 2 * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  SLNR_CUDA(cudaMemcpyAsync(A_pos2, B->pos2, ((size_t)B->nslices + 1) * sizeof(int32_t),
+                            cudaMemcpyDeviceToDevice, s));
+  if (B->nslices > 0)
+    SLNR_CUDA(cudaMemcpyAsync(A_crd1, B->crd1, (size_t)B->nslices * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  if (B->nfibers > 0)
+    SLNR_CUDA(cudaMemcpyAsync(A_crd2, B->crd2, (size_t)B->nfibers * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  if (B->nfibers == 0) return SLNR_OK;
+  const CsrView fv = fiber_view(B);
+  const SplitPlan sp = split_plan(ws, l);
+  const int tf32 = opts->allow_tf32 != 0;
+  SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
+  SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, fv, C, sp, s));
+  if (opts->variant == SLNR_FUSED) {
+    SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(L, M, fv, C, D, A_vals, tf32, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, D, M, A_vals, s));
+  } else {
+    float* T = reinterpret_cast<float*>(ws + l.o_inter);
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, fv, C, T, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
+    SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nfibers, L, M, T, D, A_vals, tf32, s));
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,148 @@
+// Inspector kernels (work decomposition for power-law inputs) and the
+// optional device-side validation of index arrays.
+//
+// The paper parallelises the shared outer sparse loop with OpenMP (Sec. 2.3,
+// Sec. 6) and names load imbalance from irregular structure as a core
+// difficulty (Sec. 1).  On the GPU the outer loop is split by nonzero count:
+// light rows are processed whole, heavy rows (more than kLightMax nonzeros)
+// are cut into chunks of kChunk nonzeros whose partial results are combined
+// in a fixed order, and MTTKRP slices are cut into windows of kUnitNnz
+// nonzeros.
+#include "launch.h"
+
+namespace slnr {
+
+int device_sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+namespace {
+
+constexpr int kErrOverflow = 8;  // inspector found more work than its bound (malformed pos)
+
+__global__ void k_classify(int nrows, const int32_t* __restrict__ pos, WsHeader* hdr,
+                           HeavyRow* __restrict__ heavy, Chunk* __restrict__ chunks, int max_heavy,
+                           int max_chunks) {
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < nrows; r += gridDim.x * blockDim.x) {
+    const int p0 = pos[r], p1 = pos[r + 1];
+    const int n = p1 - p0;
+    if (n <= kLightMax) continue;
+    const int nch = (n + kChunk - 1) / kChunk;
+    const int h = atomicAdd(&hdr->n_heavy, 1);
+    const int base = atomicAdd(&hdr->n_chunks, nch);
+    if (h >= max_heavy || base + nch > max_chunks) {
+      atomicOr(&hdr->error, kErrOverflow);
+      continue;
+    }
+    heavy[h] = HeavyRow{r, base, nch, 0};
+    for (int c = 0; c < nch; ++c) {
+      const int a = p0 + c * kChunk;
+      chunks[base + c] = Chunk{r, a, min(p1, a + kChunk), base + c};
+    }
+  }
+}
+
+__global__ void k_csf_units(int nslices, const int32_t* __restrict__ pos2,
+                            const int32_t* __restrict__ pos3, WsHeader* hdr,
+                            SliceUnits* __restrict__ su, Unit* __restrict__ units, int max_units) {
+  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < nslices; s += gridDim.x * blockDim.x) {
+    const int n = pos3[pos2[s + 1]] - pos3[pos2[s]];
+    const int nu = n > 0 ? (n + kUnitNnz - 1) / kUnitNnz : 1;
+    const int base = atomicAdd(&hdr->n_units, nu);
+    if (base + nu > max_units) {
+      atomicOr(&hdr->error, kErrOverflow);
+      su[s] = SliceUnits{0, 0};
+      continue;
+    }
+    su[s] = SliceUnits{base, nu};
+    for (int u = 0; u < nu; ++u) units[base + u] = Unit{s, u};
+  }
+}
+
+// One thread per parent: checks its position range and the order and range of
+// its children's coordinates.  Ranges are clamped so a malformed array never
+// leads to an out-of-bounds read.
+__device__ void check_level(int parent, int nparents, const int32_t* __restrict__ pos, int64_t nchild,
+                            const int32_t* __restrict__ crd, int64_t dim, int* err) {
+  const int64_t a = pos[parent], b = pos[parent + 1];
+  if (parent == 0 && a != 0) atomicOr(err, kErrPos);
+  if (parent == nparents - 1 && b != nchild) atomicOr(err, kErrPos);
+  if (a < 0 || b < a || b > nchild) {
+    atomicOr(err, kErrPos);
+    return;
+  }
+  int64_t prev = -1;
+  for (int64_t p = a; p < b; ++p) {
+    const int64_t c = crd[p];
+    if (c < 0 || c >= dim) atomicOr(err, kErrCrdRange);
+    if (c <= prev) atomicOr(err, kErrCrdOrder);
+    prev = c;
+  }
+}
+
+__global__ void k_validate_csr(slnr_csr B, WsHeader* hdr) {
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < B.nrows; r += gridDim.x * blockDim.x)
+    check_level(r, B.nrows, B.pos, B.nnz, B.crd, B.ncols, &hdr->error);
+  if (B.nrows == 0 && blockIdx.x == 0 && threadIdx.x == 0 && (B.pos[0] != 0 || B.nnz != 0))
+    atomicOr(&hdr->error, kErrPos);
+}
+
+__global__ void k_validate_csf(slnr_csf3 B, WsHeader* hdr) {
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x, nth = gridDim.x * blockDim.x;
+  if (tid == 0) {
+    if (B.pos1[0] != 0 || B.pos1[1] != B.nslices) atomicOr(&hdr->error, kErrPos);
+    if (B.nslices == 0 && (B.nfibers != 0 || B.nnz != 0)) atomicOr(&hdr->error, kErrPos);
+  }
+  for (int q = tid; q < B.nslices; q += nth) {
+    const int64_t i = B.crd1[q];
+    if (i < 0 || i >= B.dim[0]) atomicOr(&hdr->error, kErrCrdRange);
+    if (q > 0 && B.crd1[q - 1] >= i) atomicOr(&hdr->error, kErrCrdOrder);
+    check_level(q, B.nslices, B.pos2, B.nfibers, B.crd2, B.dim[1], &hdr->error);
+  }
+  for (int f = tid; f < B.nfibers; f += nth)
+    check_level(f, B.nfibers, B.pos3, B.nnz, B.crd3, B.dim[2], &hdr->error);
+}
+
+inline int grid_for(int64_t n, int block) {
+  const int64_t cap = (int64_t)device_sm_count() * 16;
+  int64_t g = (n + block - 1) / block;
+  if (g > cap) g = cap;
+  return (int)(g < 1 ? 1 : g);
+}
+
+}  // namespace
+
+cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_t s) {
+  if (B.nrows <= 0) return cudaSuccess;
+  k_classify<<<grid_for(B.nrows, 256), 256, 0, s>>>(B.nrows, B.pos, plan.hdr, plan.heavy, plan.chunks,
+                                                    plan.max_heavy, plan.max_chunks);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s) {
+  if (B.nslices <= 0) return cudaSuccess;
+  k_csf_units<<<grid_for(B.nslices, 256), 256, 0, s>>>(B.nslices, B.pos2, B.pos3, plan.hdr,
+                                                       plan.slice_units, plan.units, plan.max_units);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_validate_csr(const slnr_csr& B, WsHeader* hdr, cudaStream_t s) {
+  k_validate_csr<<<grid_for(B.nrows > 0 ? B.nrows : 1, 256), 256, 0, s>>>(B, hdr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_validate_csf(const slnr_csf3& B, WsHeader* hdr, cudaStream_t s) {
+  const int64_t n = B.nfibers > B.nslices ? B.nfibers : B.nslices;
+  k_validate_csf<<<grid_for(n > 0 ? n : 1, 256), 256, 0, s>>>(B, hdr);
+  return cudaGetLastError();
+}
+
+}  // namespace slnr

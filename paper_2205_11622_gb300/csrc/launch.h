@@ -1,0 +1,99 @@
+// Internal launchers of libslnr (C++ linkage, not exported).  Each returns
+// the cudaError_t of its launch(es); the C entry points in api.cu map them to
+// slnr_status.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace slnr {
+
+// A CSR-shaped view: rows with positions pos[nrows+1], coordinates crd and
+// values vals.  CSF fibers are viewed this way too (rows = fibers,
+// pos = pos3, crd = crd3).
+struct CsrView {
+  int nrows;
+  int ncols;
+  int64_t nnz;
+  const int32_t* pos;
+  const int32_t* crd;
+  const float* vals;
+};
+
+// Workspace pieces used to split heavy rows (see common.cuh).
+struct SplitPlan {
+  WsHeader* hdr;
+  HeavyRow* heavy;
+  Chunk* chunks;
+  float* partial;  // max_chunks x width
+  int max_heavy;
+  int max_chunks;
+};
+
+// Workspace pieces of the MTTKRP unit decomposition.
+struct UnitPlan {
+  WsHeader* hdr;
+  SliceUnits* slice_units;  // [nslices]
+  Unit* units;              // [max_units]
+  float* partial;           // max_units x L
+  int max_units;
+};
+
+int device_sm_count();
+
+// inspect.cu
+cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_t s);
+cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s);
+cudaError_t launch_validate_csr(const slnr_csr& B, WsHeader* hdr, cudaStream_t s);
+cudaError_t launch_validate_csf(const slnr_csf3& B, WsHeader* hdr, cudaStream_t s);
+
+// spmm.cu -- out[r,:] = sum_p vals[p] X[crd[p],:] (width W), and the heavy-row machinery
+cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s);
+cudaError_t launch_spmm_chunks(int W, const CsrView& B, const float* X, const SplitPlan& plan,
+                               cudaStream_t s);
+// heavy rows: out[row,:] = sum of the row's partials (width W); when D is not
+// NULL the sum (width W = K) is multiplied by D (K x L) and out has width L.
+cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, float* out,
+                           cudaStream_t s);
+
+// gemm.cu -- fused SpMM x D over light rows; dense GEMM for the unfused variant
+cudaError_t launch_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* C, const float* D,
+                                   float* A, int use_tf32, cudaStream_t s);
+cudaError_t launch_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
+                              int use_tf32, cudaStream_t s);
+
+// sddmm.cu
+cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float* D, int L,
+                                   const float* E, int K, float* A, cudaStream_t s);
+cudaError_t launch_sddmm_spmm_chunks(const CsrView& B, const float* C, const float* D, int L,
+                                     const float* E, int K, const SplitPlan& plan, cudaStream_t s);
+cudaError_t launch_sddmm_rows(const CsrView& B, const float* C, const float* D, int L, float* Y,
+                              cudaStream_t s);
+cudaError_t launch_sddmm_chunks(const CsrView& B, const float* C, const float* D, int L, float* Y,
+                                const SplitPlan& plan, cudaStream_t s);
+
+// mttkrp.cu
+cudaError_t launch_mttkrp_units(int L, const slnr_csf3& B, const float* C, const float* D,
+                                const UnitPlan& plan, cudaStream_t s);
+cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T, const float* C,
+                                       const UnitPlan& plan, cudaStream_t s);
+cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, float* A,
+                                  cudaStream_t s);
+
+}  // namespace slnr
+
+// Runs `body` with a compile-time constant WCONST equal to the runtime width
+// w (a power of two in [4, 256]); any other w returns cudaErrorInvalidValue.
+#define SLNR_WIDTH_SWITCH(w, WCONST, ...)                \
+  switch (w) {                                           \
+    case 4: { constexpr int WCONST = 4; __VA_ARGS__; } break;     \
+    case 8: { constexpr int WCONST = 8; __VA_ARGS__; } break;     \
+    case 16: { constexpr int WCONST = 16; __VA_ARGS__; } break;   \
+    case 32: { constexpr int WCONST = 32; __VA_ARGS__; } break;   \
+    case 64: { constexpr int WCONST = 64; __VA_ARGS__; } break;   \
+    case 128: { constexpr int WCONST = 128; __VA_ARGS__; } break; \
+    case 256: { constexpr int WCONST = 256; __VA_ARGS__; } break; \
+    default: return cudaErrorInvalidValue;               \
+  }

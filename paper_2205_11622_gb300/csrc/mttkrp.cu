@@ -1,0 +1,199 @@
+// MTTKRP:  A(i,l) = sum_{j,k} B(i,j,k) * C(j,l) * D(k,l),  B in CSF (i -> j -> k)
+//
+// Fused schedule (Sec. 4.2, Algorithm 1 removing C): the shared loops are the
+// slice i and the fiber j; the producer builds T(l) = sum_k B(i,j,k) D(k,l)
+// for one fiber and the consumer adds T .* C(j,:) to A(i,:) at once.  Zipf
+// slice sizes put a fifth of all nonzeros in one slice, so each slice is cut
+// into units (fibers starting in one window of kUnitNnz nonzeros); a warp
+// owns a unit, its lane groups own fibers, and each unit leaves one partial
+// A row.  k_mttkrp_combine sums a row's partials in a fixed pairwise order
+// and writes every row of A (zero for rows without a slice).
+//
+// Unfused schedule: T(f,:) for every fiber f is first written to memory
+// (spmm.cu over the fiber level), then k_mttkrp_stage2_units reads it.
+#include "launch.h"
+
+namespace slnr {
+namespace {
+
+// First f in [lo, hi) with pos[f] >= key (hi if none).
+__device__ __forceinline__ int lower_bound_pos(const int32_t* __restrict__ pos, int lo, int hi, int key) {
+  while (lo < hi) {
+    const int mid = lo + ((hi - lo) >> 1);
+    if (__ldg(pos + mid) < key) lo = mid + 1; else hi = mid;
+  }
+  return lo;
+}
+
+// Fiber range [*flo, *fhi) of unit un: the fibers of its slice whose first
+// nonzero lies in the unit's window of kUnitNnz nonzeros.
+__device__ __forceinline__ void unit_fibers(const Unit un, const SliceUnits su, const int32_t* __restrict__ pos2,
+                                            const int32_t* __restrict__ pos3, int* flo, int* fhi) {
+  const int f0 = __ldg(pos2 + un.slice), f1 = __ldg(pos2 + un.slice + 1);
+  const int start = __ldg(pos3 + f0);
+  const int lo_key = start + un.u * kUnitNnz;
+  *flo = un.u == 0 ? f0 : lower_bound_pos(pos3, f0, f1, lo_key);
+  *fhi = un.u == su.count - 1 ? f1 : lower_bound_pos(pos3, f0, f1, lo_key + kUnitNnz);
+}
+
+template <int L>
+__global__ void __launch_bounds__(256) k_mttkrp_units(const WsHeader* __restrict__ hdr,
+                                                      const Unit* __restrict__ units,
+                                                      const SliceUnits* __restrict__ sus, int max_units,
+                                                      const int32_t* __restrict__ pos2,
+                                                      const int32_t* __restrict__ crd2,
+                                                      const int32_t* __restrict__ pos3,
+                                                      const int32_t* __restrict__ crd3,
+                                                      const float* __restrict__ vals,
+                                                      const float* __restrict__ C,
+                                                      const float* __restrict__ D,
+                                                      float* __restrict__ partial) {
+  using RL = RowLanes<L>;
+  const int n = min(hdr->n_units, max_units);
+  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t w = warp; w < n; w += nwarps) {
+    const Unit un = units[w];
+    int flo, fhi;
+    unit_fibers(un, sus[un.slice], pos2, pos3, &flo, &fhi);
+    float acc[RL::VPL];
+    zero_vec(acc);
+    for (int f = flo + grp; f < fhi; f += RL::GPW) {
+      const int p0 = __ldg(pos3 + f), p1 = __ldg(pos3 + f + 1), j = __ldg(crd2 + f);
+      float c[RL::VPL];
+      ldg_vec<RL::VPL>(c, C + (int64_t)j * L + col);
+      // producer: T(l) = sum_k B(i,j,k) D(k,l), in registers
+      float t[RL::VPL];
+      zero_vec(t);
+      gather_acc<RL::VPL>(t, crd3, vals, p0, p1, D, L, col);
+      // consumer: A(i,l) += T(l) C(j,l)
+#pragma unroll
+      for (int x = 0; x < RL::VPL; ++x) acc[x] = fmaf(t[x], c[x], acc[x]);
+    }
+    cross_group_sum<RL::GS>(acc);
+    if (grp == 0) st_vec(partial + w * L + col, acc);
+  }
+}
+
+template <int L>
+__global__ void __launch_bounds__(256) k_mttkrp_stage2_units(const WsHeader* __restrict__ hdr,
+                                                             const Unit* __restrict__ units,
+                                                             const SliceUnits* __restrict__ sus, int max_units,
+                                                             const int32_t* __restrict__ pos2,
+                                                             const int32_t* __restrict__ crd2,
+                                                             const int32_t* __restrict__ pos3,
+                                                             const float* __restrict__ T,
+                                                             const float* __restrict__ C,
+                                                             float* __restrict__ partial) {
+  using RL = RowLanes<L>;
+  const int n = min(hdr->n_units, max_units);
+  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t w = warp; w < n; w += nwarps) {
+    const Unit un = units[w];
+    int flo, fhi;
+    unit_fibers(un, sus[un.slice], pos2, pos3, &flo, &fhi);
+    float acc[RL::VPL];
+    zero_vec(acc);
+    for (int f = flo + grp; f < fhi; f += RL::GPW) {
+      const int j = __ldg(crd2 + f);
+      float c[RL::VPL], t[RL::VPL];
+      ldg_vec<RL::VPL>(c, C + (int64_t)j * L + col);
+      ldg_vec<RL::VPL>(t, T + (int64_t)f * L + col);
+#pragma unroll
+      for (int x = 0; x < RL::VPL; ++x) acc[x] = fmaf(t[x], c[x], acc[x]);
+    }
+    cross_group_sum<RL::GS>(acc);
+    if (grp == 0) st_vec(partial + w * L + col, acc);
+  }
+}
+
+// One CTA per output row i: find i's slice, sum its units' partials (strided
+// lanes, then a fixed pairwise tree), write A(i,:) (zeros without a slice).
+template <int L>
+__global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, const int32_t* __restrict__ crd1,
+                                                        const SliceUnits* __restrict__ sus,
+                                                        const float* __restrict__ partial,
+                                                        float* __restrict__ A) {
+  constexpr int NC = L / 4;
+  constexpr int NR = 256 / NC;
+  __shared__ float4 red[256];
+  const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
+  for (int i = blockIdx.x; i < d0; i += gridDim.x) {
+    int lo = 0, hi = nslices;  // first slice with crd1 >= i
+    while (lo < hi) {
+      const int mid = lo + ((hi - lo) >> 1);
+      if (__ldg(crd1 + mid) < i) lo = mid + 1; else hi = mid;
+    }
+    int base = 0, count = 0;
+    if (lo < nslices && __ldg(crd1 + lo) == i) {
+      const SliceUnits su = sus[lo];
+      base = su.base;
+      count = su.count;
+    }
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int u = rl; u < count; u += NR) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(base + u) * L) + c4);
+      s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+    }
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int half = NR / 2; half > 0; half >>= 1) {
+      if (rl < half) {
+        const float4 o = red[(rl + half) * NC + c4];
+        float4 m = red[rl * NC + c4];
+        m.x += o.x; m.y += o.y; m.z += o.z; m.w += o.w;
+        red[rl * NC + c4] = m;
+      }
+      __syncthreads();
+    }
+    if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
+    __syncthreads();
+  }
+}
+
+inline int grid_units(int64_t max_units) {
+  int64_t ctas = (max_units + 7) / 8;
+  const int64_t cap = (int64_t)device_sm_count() * 32;
+  if (ctas > cap) ctas = cap;
+  return (int)(ctas < 1 ? 1 : ctas);
+}
+
+}  // namespace
+
+cudaError_t launch_mttkrp_units(int L, const slnr_csf3& B, const float* C, const float* D,
+                                const UnitPlan& plan, cudaStream_t s) {
+  if (plan.max_units <= 0 || B.nslices <= 0) return cudaSuccess;
+  SLNR_WIDTH_SWITCH(L, W, {
+    k_mttkrp_units<W><<<grid_units(plan.max_units), 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units,
+                                                                 plan.max_units, B.pos2, B.crd2, B.pos3,
+                                                                 B.crd3, B.vals, C, D, plan.partial);
+  });
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T, const float* C,
+                                       const UnitPlan& plan, cudaStream_t s) {
+  if (plan.max_units <= 0 || B.nslices <= 0) return cudaSuccess;
+  SLNR_WIDTH_SWITCH(L, W, {
+    k_mttkrp_stage2_units<W><<<grid_units(plan.max_units), 256, 0, s>>>(
+        plan.hdr, plan.units, plan.slice_units, plan.max_units, B.pos2, B.crd2, B.pos3, T, C, plan.partial);
+  });
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, float* A,
+                                  cudaStream_t s) {
+  if (B.dim[0] <= 0) return cudaSuccess;
+  int grid = B.dim[0];
+  const int cap = device_sm_count() * 8;
+  if (grid > cap) grid = cap;
+  SLNR_WIDTH_SWITCH(L, W, {
+    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.dim[0], B.nslices, B.crd1, plan.slice_units, plan.partial, A);
+  });
+  return cudaGetLastError();
+}
+
+}  // namespace slnr

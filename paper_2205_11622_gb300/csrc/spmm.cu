@@ -1,0 +1,152 @@
+// Sparse-times-dense producer stages and the heavy-row combine.
+//
+//   out[r,:] = sum_{p in row r} vals[p] * X[crd[p], :]        (width W)
+//
+// This is the SpMM of Fig. 2b and the producer of <SpMM,GEMM> (T = B.C),
+// of <SpTTM,SpTTM> (T = B x_3 C per fiber) and of MTTKRP's unfused variant.
+// A group of lanes owns one row (common.cuh, RowLanes), so light rows need no
+// cross-lane reduction; heavy rows go through chunks and k_combine.
+#include "launch.h"
+
+namespace slnr {
+namespace {
+
+template <int W>
+__global__ void __launch_bounds__(256) k_spmm_rows(int nrows, const int32_t* __restrict__ pos,
+                                                   const int32_t* __restrict__ crd,
+                                                   const float* __restrict__ vals,
+                                                   const float* __restrict__ X, float* __restrict__ out) {
+  using RL = RowLanes<W>;
+  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t r = warp * RL::GPW + grp; r < nrows; r += nwarps * RL::GPW) {
+    const int p0 = pos[r], p1 = pos[r + 1];
+    if (p1 - p0 > kLightMax) continue;  // written by the heavy-row path
+    float acc[RL::VPL];
+    zero_vec(acc);
+    gather_acc<RL::VPL>(acc, crd, vals, p0, p1, X, W, col);
+    st_vec(out + r * W + col, acc);
+  }
+}
+
+template <int W>
+__global__ void __launch_bounds__(256) k_spmm_chunks(const WsHeader* __restrict__ hdr,
+                                                     const Chunk* __restrict__ chunks, int max_chunks,
+                                                     const int32_t* __restrict__ crd,
+                                                     const float* __restrict__ vals,
+                                                     const float* __restrict__ X,
+                                                     float* __restrict__ partial) {
+  using RL = RowLanes<W>;
+  const int n = min(hdr->n_chunks, max_chunks);
+  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t c = warp * RL::GPW + grp; c < n; c += nwarps * RL::GPW) {
+    const Chunk ch = chunks[c];
+    float acc[RL::VPL];
+    zero_vec(acc);
+    gather_acc<RL::VPL>(acc, crd, vals, ch.p0, ch.p1, X, W, col);
+    st_vec(partial + (int64_t)ch.slot * W + col, acc);
+  }
+}
+
+// One CTA per heavy row: the row's partials (width W) are summed by
+// kRowLanes lanes each taking every kRowLanes-th partial, then by a fixed
+// pairwise tree, so the result does not depend on scheduling and long rows
+// keep a short rounding chain.  With D, the sum t (length W = K) is then
+// multiplied by D (K x L): out[row, l] = sum_k t[k] D[k, l].
+template <int W>
+__global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hdr,
+                                                 const HeavyRow* __restrict__ heavy, int max_heavy,
+                                                 const float* __restrict__ partial,
+                                                 const float* __restrict__ D, int L,
+                                                 float* __restrict__ out) {
+  constexpr int NC = W / 4;                 // float4 columns
+  constexpr int NR = 256 / NC;              // lanes along the partials
+  __shared__ float4 red[256];
+  __shared__ float t[W];
+  const int n = min(hdr->n_heavy, max_heavy);
+  const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
+  for (int h = blockIdx.x; h < n; h += gridDim.x) {
+    const HeavyRow hr = heavy[h];
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (rl < NR) {
+      for (int c = rl; c < hr.count; c += NR) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(hr.base + c) * W) + c4);
+        s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+      }
+    }
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int half = NR / 2; half > 0; half >>= 1) {
+      if (rl < half) {
+        const float4 o = red[(rl + half) * NC + c4];
+        float4 m = red[rl * NC + c4];
+        m.x += o.x; m.y += o.y; m.z += o.z; m.w += o.w;
+        red[rl * NC + c4] = m;
+      }
+      __syncthreads();
+    }
+    if (D == nullptr) {
+      if (rl == 0) reinterpret_cast<float4*>(out + (int64_t)hr.row * W)[c4] = red[c4];
+    } else {
+      if (rl == 0) {
+        const float4 v = red[c4];
+        t[4 * c4 + 0] = v.x; t[4 * c4 + 1] = v.y; t[4 * c4 + 2] = v.z; t[4 * c4 + 3] = v.w;
+      }
+      __syncthreads();
+      for (int l = threadIdx.x; l < L; l += blockDim.x) {
+        float acc = 0.f;
+#pragma unroll 8
+        for (int k = 0; k < W; ++k) acc = fmaf(t[k], __ldg(D + (int64_t)k * L + l), acc);
+        out[(int64_t)hr.row * L + l] = acc;
+      }
+    }
+    __syncthreads();
+  }
+}
+
+inline int grid_warps(int64_t items_per_warp_round, int64_t n) {
+  // enough CTAs of 8 warps to cover n items (items_per_warp_round per warp),
+  // capped at 32 CTAs per SM; grid-stride loops cover the rest
+  int64_t warps = (n + items_per_warp_round - 1) / items_per_warp_round;
+  int64_t ctas = (warps + 7) / 8;
+  const int64_t cap = (int64_t)device_sm_count() * 32;
+  if (ctas > cap) ctas = cap;
+  return (int)(ctas < 1 ? 1 : ctas);
+}
+
+}  // namespace
+
+cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s) {
+  if (B.nrows <= 0) return cudaSuccess;
+  SLNR_WIDTH_SWITCH(W, WC, {
+    k_spmm_rows<WC><<<grid_warps(RowLanes<WC>::GPW, B.nrows), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, out);
+  });
+  return cudaGetLastError();
+}
+
+cudaError_t launch_spmm_chunks(int W, const CsrView& B, const float* X, const SplitPlan& plan,
+                               cudaStream_t s) {
+  if (plan.max_chunks <= 0) return cudaSuccess;
+  SLNR_WIDTH_SWITCH(W, WC, {
+    k_spmm_chunks<WC><<<grid_warps(RowLanes<WC>::GPW, plan.max_chunks), 256, 0, s>>>(
+        plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X, plan.partial);
+  });
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, float* out,
+                           cudaStream_t s) {
+  if (plan.max_heavy <= 0) return cudaSuccess;
+  int grid = plan.max_heavy;
+  const int cap = device_sm_count() * 8;
+  if (grid > cap) grid = cap;
+  SLNR_WIDTH_SWITCH(W, WC, {
+    k_combine<WC><<<grid, 256, 0, s>>>(plan.hdr, plan.heavy, plan.max_heavy, plan.partial, D, L, out);
+  });
+  return cudaGetLastError();
+}
+
+}  // namespace slnr
