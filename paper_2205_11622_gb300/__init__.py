@@ -235,6 +235,19 @@ class Workspace:
 
 
 _default_ws = {}
+_last_ws = [None]
+
+# Bits of the device-side flag word (offset 12 of the workspace header).
+DEVICE_FLAGS = {1: "position array malformed", 2: "coordinate out of range", 4: "coordinates not increasing",
+                8: "inspector bound exceeded", 16: "device wait timed out"}
+
+
+def device_flags(workspace=None) -> int:
+    """Flag word the kernels of the last call on this workspace set (0 = none); synchronises."""
+    buf = workspace.buf if workspace is not None else _last_ws[0]
+    if buf is None:
+        return 0
+    return int(buf[12:16].view(_torch().int32).item())
 
 
 def _opts(variant, allow_tf32, validate, stream):
@@ -250,6 +263,7 @@ def _attach_ws(opts, nbytes, workspace):
         dev = torch.cuda.current_device()
         workspace = _default_ws.setdefault((dev, opts.stream), Workspace(device=f"cuda:{dev}"))
     buf = workspace.get(nbytes)
+    _last_ws[0] = buf
     opts.workspace = buf.data_ptr()
     opts.workspace_bytes = buf.numel()
     return buf

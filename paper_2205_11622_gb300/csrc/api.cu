@@ -89,6 +89,24 @@ struct Layout {
     o_units = take(sizeof(Unit) * (size_t)max_units);
     o_upartial = take(sizeof(float) * (size_t)max_units * (size_t)width);
   }
+  // row segments of the tensor-core path (partials are A rows of the output width)
+  size_t o_counts = 0, o_segs = 0;
+  int max_segs = 0;
+  void segs(int64_t nrows, int64_t nnz, int width) {
+    int64_t mh = 0, mc = 0;
+    if (nnz > kSegChunk) {
+      mh = nnz / (kSegChunk + 1);
+      if (mh > nrows) mh = nrows;
+      mc = nnz / kSegChunk + mh + 1;
+    }
+    max_heavy = (int)mh;
+    max_chunks = (int)mc;
+    max_segs = (int)(nrows + mc);
+    o_counts = take(sizeof(int) * 3 * (size_t)seg_scan_blocks(nrows));
+    o_segs = take(sizeof(int4) * (size_t)max_segs);
+    o_heavy = take(sizeof(HeavyRow) * (size_t)mh);
+    o_partial = take(sizeof(float) * (size_t)mc * (size_t)width);
+  }
   size_t o_inter = 0;
   void inter(size_t bytes) { o_inter = take(bytes); }
   size_t total() const { return align256(cur); }
@@ -98,6 +116,17 @@ SplitPlan split_plan(char* ws, const Layout& l) {
   return SplitPlan{reinterpret_cast<WsHeader*>(ws), reinterpret_cast<HeavyRow*>(ws + l.o_heavy),
                    reinterpret_cast<Chunk*>(ws + l.o_chunks), reinterpret_cast<float*>(ws + l.o_partial),
                    l.max_heavy, l.max_chunks};
+}
+
+SegPlan seg_plan(char* ws, const Layout& l) {
+  return SegPlan{reinterpret_cast<WsHeader*>(ws), reinterpret_cast<int*>(ws + l.o_counts),
+                 reinterpret_cast<int4*>(ws + l.o_segs), reinterpret_cast<HeavyRow*>(ws + l.o_heavy),
+                 reinterpret_cast<float*>(ws + l.o_partial), l.max_segs, l.max_heavy, l.max_chunks};
+}
+
+// The heavy-row records and partial rows of a segment plan, as k_combine reads them.
+SplitPlan combine_plan(const SegPlan& g) {
+  return SplitPlan{g.hdr, g.heavy, nullptr, g.partial, g.max_heavy, g.max_chunks};
 }
 
 UnitPlan unit_plan(char* ws, const Layout& l) {
@@ -198,11 +227,17 @@ slnr_status begin(char* ws, cudaStream_t s, bool validate, Launch launch_validat
 // ---------------------------------------------------------------------------
 // layouts per operation
 
-Layout layout_spmm_gemm(const slnr_csr* B, int32_t K, int32_t L, int variant) {
-  (void)L;
+// The fused tensor-core path takes row segments; everything else splits heavy rows.
+bool use_tc(const slnr_opts* o, int32_t K, int32_t L) { return o->allow_tf32 != 0 && tc_supported(K, L); }
+
+Layout layout_spmm_gemm(const slnr_csr* B, int32_t K, int32_t L, const slnr_opts* o) {
   Layout l;
-  l.split(B->nrows, B->nnz, K);
-  if (variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nrows * (size_t)K);
+  if (o->variant == SLNR_FUSED && use_tc(o, K, L)) {
+    l.segs(B->nrows, B->nnz, L);
+  } else {
+    l.split(B->nrows, B->nnz, K);
+    if (o->variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nrows * (size_t)K);
+  }
   return l;
 }
 
@@ -224,11 +259,14 @@ Layout layout_mttkrp(const slnr_csf3* B, int32_t L, int variant) {
   return l;
 }
 
-Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, int variant) {
-  (void)M;
+Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opts* o) {
   Layout l;
-  l.split(B->nfibers, B->nnz, L);
-  if (variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nfibers * (size_t)L);
+  if (o->variant == SLNR_FUSED && use_tc(o, L, M)) {
+    l.segs(B->nfibers, B->nnz, M);
+  } else {
+    l.split(B->nfibers, B->nnz, L);
+    if (o->variant == SLNR_UNFUSED) l.inter(sizeof(float) * (size_t)B->nfibers * (size_t)L);
+  }
   return l;
 }
 
@@ -289,7 +327,7 @@ slnr_status slnr_spmm_gemm_workspace(const slnr_csr* B, int32_t K, int32_t L, co
   SLNR_CHECK(check_dims("K", K));
   SLNR_CHECK(check_dims("L", L));
   if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
-  *bytes = layout_spmm_gemm(B, K, L, opts->variant).total();
+  *bytes = layout_spmm_gemm(B, K, L, opts).total();
   return SLNR_OK;
 }
 
@@ -320,7 +358,7 @@ slnr_status slnr_spttm_ttm_workspace(const slnr_csf3* B, int32_t L, int32_t M, c
   SLNR_CHECK(check_dims("L", L));
   SLNR_CHECK(check_dims("M", M));
   if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
-  *bytes = layout_spttm_ttm(B, L, M, opts->variant).total();
+  *bytes = layout_spttm_ttm(B, L, M, opts).total();
   return SLNR_OK;
 }
 
@@ -335,7 +373,7 @@ slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const f
   SLNR_CHECK(check_dense("C", C));
   SLNR_CHECK(check_dense("D", D));
   SLNR_CHECK(check_dense("A", A));
-  const Layout l = layout_spmm_gemm(B, K, L, opts->variant);
+  const Layout l = layout_spmm_gemm(B, K, L, opts);
   SLNR_CHECK(check_ws(opts, l.total()));
   if (B->nrows == 0) return SLNR_OK;
   cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
@@ -343,18 +381,29 @@ slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const f
   SLNR_CHECK(begin(ws, s, opts->validate != 0,
                    [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
   const CsrView v = csr_view(B);
-  const SplitPlan sp = split_plan(ws, l);
-  const int tf32 = opts->allow_tf32 != 0;
-  SLNR_LAUNCH("classify", launch_classify(v, sp, s));
-  SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(K, v, C, sp, s));
-  if (opts->variant == SLNR_FUSED) {
-    SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(K, L, v, C, D, A, tf32, s));
-    SLNR_LAUNCH("combine", launch_combine(K, sp, D, L, A, s));
+  const bool tc = use_tc(opts, K, L);
+  if (opts->variant == SLNR_FUSED && tc) {
+    const SegPlan gp = seg_plan(ws, l);
+    SLNR_LAUNCH("seg_count", launch_seg_count(v, gp, s));
+    SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
+    SLNR_LAUNCH("tc_spmm_gemm", launch_tc_spmm_gemm(K, L, v, C, D, A, gp, s));
+    SLNR_LAUNCH("combine", launch_combine(L, combine_plan(gp), nullptr, 0, A, s));
   } else {
-    float* T = reinterpret_cast<float*>(ws + l.o_inter);
-    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(K, v, C, T, s));
-    SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, T, s));
-    SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, K, L, T, D, A, tf32, s));
+    const SplitPlan sp = split_plan(ws, l);
+    SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(K, v, C, sp, s));
+    if (opts->variant == SLNR_FUSED) {
+      SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(K, L, v, C, D, A, 0, s));
+      SLNR_LAUNCH("combine", launch_combine(K, sp, D, L, A, s));
+    } else {
+      float* T = reinterpret_cast<float*>(ws + l.o_inter);
+      SLNR_LAUNCH("spmm_rows", launch_spmm_rows(K, v, C, T, s));
+      SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, T, s));
+      if (tc)
+        SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nrows, K, L, T, D, A, sp.hdr, s));
+      else
+        SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, K, L, T, D, A, 0, s));
+    }
   }
   timing_end(s);
   return SLNR_OK;
@@ -450,7 +499,7 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
   if (!A_pos1 || !A_pos2 || (B->nslices > 0 && !A_crd1) || (B->nfibers > 0 && !A_crd2))
     return fail(SLNR_ERR_NULL, "an output index array of A is NULL");
   if (B->nfibers > 0) SLNR_CHECK(check_dense("A_vals", A_vals));
-  const Layout l = layout_spttm_ttm(B, L, M, opts->variant);
+  const Layout l = layout_spttm_ttm(B, L, M, opts);
   SLNR_CHECK(check_ws(opts, l.total()));
   cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
   char* ws = static_cast<char*>(opts->workspace);
@@ -466,18 +515,29 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
     SLNR_CUDA(cudaMemcpyAsync(A_crd2, B->crd2, (size_t)B->nfibers * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
   if (B->nfibers == 0) return SLNR_OK;
   const CsrView fv = fiber_view(B);
-  const SplitPlan sp = split_plan(ws, l);
-  const int tf32 = opts->allow_tf32 != 0;
-  SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
-  SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, fv, C, sp, s));
-  if (opts->variant == SLNR_FUSED) {
-    SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(L, M, fv, C, D, A_vals, tf32, s));
-    SLNR_LAUNCH("combine", launch_combine(L, sp, D, M, A_vals, s));
+  const bool tc = use_tc(opts, L, M);
+  if (opts->variant == SLNR_FUSED && tc) {
+    const SegPlan gp = seg_plan(ws, l);
+    SLNR_LAUNCH("seg_count", launch_seg_count(fv, gp, s));
+    SLNR_LAUNCH("seg_write", launch_seg_write(fv, gp, s));
+    SLNR_LAUNCH("tc_spmm_gemm", launch_tc_spmm_gemm(L, M, fv, C, D, A_vals, gp, s));
+    SLNR_LAUNCH("combine", launch_combine(M, combine_plan(gp), nullptr, 0, A_vals, s));
   } else {
-    float* T = reinterpret_cast<float*>(ws + l.o_inter);
-    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, fv, C, T, s));
-    SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
-    SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nfibers, L, M, T, D, A_vals, tf32, s));
+    const SplitPlan sp = split_plan(ws, l);
+    SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, fv, C, sp, s));
+    if (opts->variant == SLNR_FUSED) {
+      SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(L, M, fv, C, D, A_vals, 0, s));
+      SLNR_LAUNCH("combine", launch_combine(L, sp, D, M, A_vals, s));
+    } else {
+      float* T = reinterpret_cast<float*>(ws + l.o_inter);
+      SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, fv, C, T, s));
+      SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
+      if (tc)
+        SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nfibers, L, M, T, D, A_vals, sp.hdr, s));
+      else
+        SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nfibers, L, M, T, D, A_vals, 0, s));
+    }
   }
   timing_end(s);
   return SLNR_OK;

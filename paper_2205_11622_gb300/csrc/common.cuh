@@ -22,13 +22,16 @@ constexpr int kChunk = 256;
 // MTTKRP: a slice is cut into units of fibers that start within one window
 // of kUnitNnz nonzeros.
 constexpr int kUnitNnz = 512;
+// Tensor-core path: rows are cut into segments of at most kSegChunk nonzeros.
+constexpr int kSegChunk = 128;
 
 struct WsHeader {        // first 256 bytes of every workspace
   int n_heavy;           // heavy rows found by the inspector
   int n_chunks;          // chunks of heavy rows
   int n_units;           // MTTKRP units
-  int error;             // validation flags (bit set = problem found)
-  int pad[60];
+  int error;             // validation / runtime flags (bit set = problem found)
+  int n_segs;            // segments of the tensor-core path
+  int pad[59];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 
@@ -61,6 +64,8 @@ enum : int {
   kErrPos = 1,          // position array not monotone / wrong ends
   kErrCrdRange = 2,     // coordinate out of range
   kErrCrdOrder = 4,     // coordinates not strictly increasing in a parent
+  kErrOverflow = 8,     // inspector found more work than its bound (malformed positions)
+  kErrTimeout = 16,     // a bounded device-side wait gave up
 };
 
 // ---------------------------------------------------------------------------

@@ -127,9 +127,11 @@ __global__ void __launch_bounds__(256) k_dense_gemm(int64_t M, const float* __re
   tile_times_d<K>(T, D, L, Ds, A, r0, M, nullptr);
 }
 
+// Opt in to more than the default 48 KB of dynamic shared memory (the
+// kernels also hold a little static shared memory).
 template <typename Kern>
 cudaError_t set_smem(Kern k, size_t bytes) {
-  if (bytes <= 48 * 1024) return cudaSuccess;
+  if (bytes <= 40 * 1024) return cudaSuccess;
   return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 

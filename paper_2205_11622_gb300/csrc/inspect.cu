@@ -26,8 +26,6 @@ int device_sm_count() {
 
 namespace {
 
-constexpr int kErrOverflow = 8;  // inspector found more work than its bound (malformed pos)
-
 __global__ void k_classify(int nrows, const int32_t* __restrict__ pos, WsHeader* hdr,
                            HeavyRow* __restrict__ heavy, Chunk* __restrict__ chunks, int max_heavy,
                            int max_chunks) {

@@ -41,6 +41,19 @@ struct UnitPlan {
   int max_units;
 };
 
+// Workspace pieces of the tensor-core path: row segments of at most
+// kSegChunk nonzeros (tc_gemm.cu).
+struct SegPlan {
+  WsHeader* hdr;
+  int* block_counts;  // 3 ints per inspector block
+  int4* segs;         // {row, p0, p1, partial slot or -1}
+  HeavyRow* heavy;
+  float* partial;     // max_chunks x L partial A rows
+  int max_segs;
+  int max_heavy;
+  int max_chunks;
+};
+
 int device_sm_count();
 
 // inspect.cu
@@ -63,6 +76,16 @@ cudaError_t launch_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* 
                                    float* A, int use_tf32, cudaStream_t s);
 cudaError_t launch_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                               int use_tf32, cudaStream_t s);
+
+// tc_gemm.cu -- tcgen05 TF32 consumer contraction
+bool tc_supported(int K, int L);
+int seg_scan_blocks(int64_t nrows);
+cudaError_t launch_seg_count(const CsrView& B, const SegPlan& plan, cudaStream_t s);
+cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t s);
+cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, const float* D, float* A,
+                                const SegPlan& plan, cudaStream_t s);
+cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
+                                 WsHeader* hdr, cudaStream_t s);
 
 // sddmm.cu
 cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float* D, int L,
