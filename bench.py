@@ -238,7 +238,7 @@ def dist_env():
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
-    ws = [wl.full(i) for i in BENCH_CONFIGS]
+    ws = select_workloads(args)
     budget = args.ref_gflop_per_expr * 1e9
     times, flops_total, sample = [], 0, ""
     for step in range(args.warmup + args.steps):
@@ -264,6 +264,14 @@ def run_reference(args, rank, world):
     return 0
 
 
+def select_workloads(args):
+    ws = [wl.full(i, args.scale) for i in BENCH_CONFIGS]
+    ws = [w for w in ws if args.expr in w.name]
+    if not ws:
+        raise SystemExit(f"no workload matches --expr {args.expr!r}")
+    return ws
+
+
 def config_block(ws):
     return {
         "workload": " + ".join(w.name for w in ws),
@@ -286,6 +294,8 @@ def main():
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-gflop-per-expr", type=float, default=4.0)
     ap.add_argument("--ref-gflop-per-expr", type=float, default=1.0)
+    ap.add_argument("--expr", default="", help="only the expressions whose name contains this (profiling)")
+    ap.add_argument("--scale", type=float, default=1.0, help="shrink the workloads (profiling captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -308,7 +318,7 @@ def main():
     slnr.lib()
     allow_tf32 = not args.no_tf32
 
-    ws = [wl.full(i) for i in BENCH_CONFIGS]
+    ws = select_workloads(args)
     flops = [useful_flops(w) for w in ws]
     mbytes = [min_bytes(w) for w in ws]
 

@@ -285,20 +285,24 @@ def spttm_ttm_powerlaw(seed: int, dims, nnz: int, mean_len: float, max_len: int,
                     f"seed {seed:#x}")
 
 
-# The five benchmark workloads at full size (index = position in the benchmark list).
-def full(index: int) -> Workload:
+# The five benchmark workloads at full size (index = position in the benchmark
+# list).  `scale` < 1 shrinks the row count (R-MAT) or the nonzero count (CSF)
+# with the same recipe, for profiling captures on smaller cases.
+def full(index: int, scale: float = 1.0) -> Workload:
     seed = SEED_BASE + index
+    tag = "" if scale == 1.0 else f"_x{scale:g}"
     if index == 0:
         return spmm_gemm_uniform(seed, 1024, 1024, 10, 32, 32, name="spmm_gemm_1k_k32")
     if index == 1:
-        return sddmm_spmm_rmat(seed, 100_000, 20, 64, 64, name="sddmm_spmm_rmat100k_d20_64")
+        return sddmm_spmm_rmat(seed, int(100_000 * scale), 20, 64, 64, name="sddmm_spmm_rmat100k_d20_64" + tag)
     if index == 2:
-        return spmm_gemm_rmat(seed, 1 << 20, 16, 128, 128, name="spmm_gemm_rmat1m_d16_k128")
+        return spmm_gemm_rmat(seed, int((1 << 20) * scale), 16, 128, 128, name="spmm_gemm_rmat1m_d16_k128" + tag)
     if index == 3:
-        return mttkrp_zipf(seed, (10_000, 10_000, 10_000), 10_000_000, 1.2, 32, name="mttkrp_zipf10k_10m_l32")
+        return mttkrp_zipf(seed, (10_000, 10_000, 10_000), int(10_000_000 * scale), 1.2, 32,
+                           name="mttkrp_zipf10k_10m_l32" + tag)
     if index == 4:
-        return spttm_ttm_powerlaw(seed, (5_000, 5_000, 5_000), 20_000_000, 8.0, 5_000, 64, 64,
-                                  name="spttm_ttm_powerlaw5k_20m_64")
+        return spttm_ttm_powerlaw(seed, (5_000, 5_000, 5_000), int(20_000_000 * scale), 8.0, 5_000, 64, 64,
+                                  name="spttm_ttm_powerlaw5k_20m_64" + tag)
     raise IndexError(index)
 
 
