@@ -160,6 +160,25 @@ slnr_status slnr_spttm_ttm(const slnr_csf3 *B, const float *C, int32_t L, const 
                            int32_t *A_pos1, int32_t *A_crd1, int32_t *A_pos2, int32_t *A_crd2,
                            float *A_vals, const slnr_opts *opts);
 
+/* ---- <SDDMM,SpMM> without a caller workspace ----------------------------
+ * The paper has no counterpart to this entry point; it serves callers that
+ * cannot allocate device memory (code inside a CUDA graph being captured, a
+ * real-time or signal-safe path that must not enter an allocator, or a host
+ * runtime that owns all device memory).  It runs the fused variant of
+ * slnr_sddmm_spmm with the same arguments and results, but its scratch is a
+ * 16 MiB array inside the library's device code: every GPU that loads the
+ * library holds those 16 MiB until the process exits, and the call allocates
+ * nothing.  Sizes whose scratch would exceed 16 MiB (about 7 million nonzeros
+ * at K = 64) return SLNR_ERR_UNSUPPORTED.  The first call on each device
+ * looks up the array's device address (cudaGetSymbolAddress) with that device
+ * current; make that first call before any stream capture begins.  All calls
+ * share the one array: the call clears what must start at zero itself, and
+ * calls whose work overlaps on the GPU (other streams, other host threads)
+ * race on it.  Runs on `stream` (a cudaStream_t, NULL = legacy default), with
+ * validate off and fp32 arithmetic. */
+slnr_status slnr_sddmm_spmm_noalloc(const slnr_csr *B, const float *C, const float *D, int32_t L,
+                                    const float *E, int32_t K, float *A, void *stream);
+
 /* ---- per-launch timing (instrumentation) --------------------------------
  * With timing enabled, each call on the calling thread records a CUDA event on
  * opts->stream before each of its kernel launches and one after the last, so

@@ -64,6 +64,7 @@ SIGNATURES = {
     "slnr_sddmm_spmm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_mttkrp": ([_CSF, _P, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_spttm_ttm": ([_CSF, _P, _I32, _P, _I32, _P, _P, _P, _P, _P, _OPT], ctypes.c_int),
+    "slnr_sddmm_spmm_noalloc": ([_CSR, _P, _P, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
     "slnr_timing_get": ([_I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),

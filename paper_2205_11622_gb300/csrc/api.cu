@@ -277,6 +277,8 @@ CsrView fiber_view(const slnr_csf3* B) {
 
 }  // namespace
 
+void slnr::set_last_error(const char* msg) { snprintf(g_last_error, sizeof(g_last_error), "%s", msg); }
+
 // ===========================================================================
 
 extern "C" {

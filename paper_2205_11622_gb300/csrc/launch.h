@@ -56,6 +56,9 @@ struct SegPlan {
 
 int device_sm_count();
 
+// Sets the calling thread's slnr_last_error() text (api.cu).
+void set_last_error(const char* msg);
+
 // inspect.cu
 cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_t s);
 cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s);
