@@ -26,7 +26,7 @@ namespace slnr {
 
 namespace {
 
-constexpr int kTcThreads = 512;
+constexpr int kTcThreads = 1024;
 constexpr int kTcRows = 128;  // MMA M
 constexpr int kScanRows = 2048;
 constexpr int kScanThreads = 256;
@@ -159,6 +159,14 @@ __global__ void __launch_bounds__(kScanThreads) k_seg_write(int nrows, const int
   }
 }
 
+// Waits until *count >= target (a monotonic shared-memory counter); false on timeout.
+__device__ __forceinline__ bool count_wait_timeout(const int* count, int target) {
+  const long long t0 = clock64();
+  while (tc::ld_acquire_smem(count) < target)
+    if (clock64() - t0 > kWaitCycles) return false;
+  return true;
+}
+
 __device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity) {
   const long long t0 = clock64();
   while (!tc::mbar_try_wait(bar, parity))
@@ -168,11 +176,142 @@ __device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity
 
 enum TcMode { kSegments = 0, kDense = 1 };
 
-// Shared memory: T tile (kTcRows x K) and D^T (L x K), both tf32 K-major
+// Number of T / accumulator buffers: up to four, as many as fit beside D^T
+// in shared memory (200 KB budget) and in tensor memory (512 columns).
+__host__ __device__ constexpr int tc_nbuf(int K, int L) {
+  return ((size_t)4 * kTcRows * K * 4 + (size_t)L * K * 4 + 1024 <= (size_t)200 * 1024 && 4 * L <= 512) ? 4 : 2;
+}
+
+// Shared memory: NBUF T tiles (kTcRows x K) and D^T (L x K), tf32 K-major
 // 128B-swizzled, plus 1 KB of alignment slack.
 __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
-  return (size_t)kTcRows * K * 4 + (size_t)L * K * 4 + 1024;
+  return (size_t)tc_nbuf(K, L) * kTcRows * K * 4 + (size_t)L * K * 4 + 1024;
 }
+
+#ifndef SLNR_TC_VEC_K128
+#define SLNR_TC_VEC_K128 1  // float4 per lane, K = 128
+#endif
+#ifndef SLNR_TC_U_K128
+#define SLNR_TC_U_K128 4    // rows in flight per group, K = 128
+#endif
+#ifndef SLNR_TC_VEC_K64
+#define SLNR_TC_VEC_K64 1   // float4 per lane, K <= 64
+#endif
+#ifndef SLNR_TC_U_K64
+#define SLNR_TC_U_K64 4     // rows in flight per group, K <= 64
+#endif
+
+// Lane layout of the producer: a group of GS lanes builds T rows; lane gl
+// holds VEC float4 of a row, at columns 4*gl + v*(K/VEC) (v < VEC), and
+// keeps U gathered rows of X in flight.  A claim is kQuad consecutive items
+// (segments), whose nonzeros form one contiguous range.
+template <int K>
+struct ProdLayout {
+  static constexpr int VEC = K >= 128 ? SLNR_TC_VEC_K128 : SLNR_TC_VEC_K64;
+  static constexpr int GS = K / (4 * VEC);
+  static constexpr int U = K >= 128 ? SLNR_TC_U_K128 : SLNR_TC_U_K64;
+};
+constexpr int kQuad = 4;
+
+template <int VEC>
+__device__ __forceinline__ void store_t_row(uint8_t* sTb, int s, int gl, int K, const float4 (&acc)[VEC]) {
+#pragma unroll
+  for (int w = 0; w < VEC; ++w)
+    *reinterpret_cast<uint4*>(sTb + tc::sw128_offset(s, 4 * gl + w * (K / VEC), kTcRows)) =
+        make_uint4(tc::to_tf32(acc[w].x), tc::to_tf32(acc[w].y), tc::to_tf32(acc[w].z), tc::to_tf32(acc[w].w));
+}
+
+// Accumulates the kQuad rows of one claim: row q sums vals[p] X[crd[p],:] over
+// its range, which ends at the value lane src0+q of the group holds in my_end;
+// the ranges are consecutive from p, so one pipeline of U row gathers runs
+// over all of them, and emit(q, acc) hands each row on as soon as its range is
+// done (returns false to abandon the claim).  Coordinates and values of the
+// next batch are fetched while the current rows are in flight, each by one
+// lane of the group and passed on by shuffles.
+template <int K, int VEC, int U, typename Emit>
+__device__ __forceinline__ bool build_quad(int my_end, int p, unsigned gmask, int src0, int gl,
+                                           const int32_t* __restrict__ crd, const float* __restrict__ vals,
+                                           const float* __restrict__ X, Emit&& emit) {
+  const int p_end = __shfl_sync(gmask, my_end, src0 + kQuad - 1);
+  float4 acc[VEC];
+#pragma unroll
+  for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+  int q = 0;
+  int cur_end = __shfl_sync(gmask, my_end, src0);
+  int my_c = 0;
+  float my_v = 0.f;
+  if (gl < U && p + gl < p_end) {
+    my_c = __ldg(crd + p + gl);
+    my_v = __ldg(vals + p + gl);
+  }
+  while (p < p_end) {
+    float v[U];
+    float4 x[U][VEC];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int cu = __shfl_sync(gmask, my_c, src0 + u);
+      v[u] = __shfl_sync(gmask, my_v, src0 + u);
+      const float* row = X + (int64_t)cu * K + 4 * gl;
+#pragma unroll
+      for (int w = 0; w < VEC; ++w)
+        x[u][w] = (p + u < p_end) ? __ldg(reinterpret_cast<const float4*>(row + w * (K / VEC)))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    const int pn = p + U;
+    my_c = 0;
+    my_v = 0.f;
+    if (gl < U && pn + gl < p_end) {
+      my_c = __ldg(crd + pn + gl);
+      my_v = __ldg(vals + pn + gl);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (p + u < p_end) {
+        while (p + u >= cur_end) {  // rows whose range is complete (empty rows included)
+          if (!emit(q, acc)) return false;
+#pragma unroll
+          for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+          ++q;
+          cur_end = __shfl_sync(gmask, my_end, src0 + q);
+        }
+#pragma unroll
+        for (int w = 0; w < VEC; ++w) {
+          acc[w].x = fmaf(v[u], x[u][w].x, acc[w].x);
+          acc[w].y = fmaf(v[u], x[u][w].y, acc[w].y);
+          acc[w].z = fmaf(v[u], x[u][w].z, acc[w].z);
+          acc[w].w = fmaf(v[u], x[u][w].w, acc[w].w);
+        }
+      }
+    }
+    p = pn;
+  }
+  for (; q < kQuad; ++q) {
+    if (!emit(q, acc)) return false;
+#pragma unroll
+    for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  return true;
+}
+
+// Warp roles of the persistent tile kernel (32 warps):
+//   warps 0..26  producers: claim kQuad of this CTA's items at a time, build
+//                their T rows on chip, and put each finished row into the next
+//                free slot of the open T buffer, recording its destination;
+//                MMA tiles are thus filled in completion order, so a long
+//                segment delays only its own row, never a whole tile;
+//   warp 27      MMA issuer: waits full[b] (128 rows placed) and free[b]
+//                (buffer's previous accumulator drained), issues the tile's
+//                K/8 tcgen05.mma into TMEM accumulator b, commits to mma[b];
+//   warps 28..31 epilogue: wait mma[b], read TMEM lane quadrant (warp % 4),
+//                write A rows or partial rows, arrive free[b].
+// Slot tile n uses buffer n % NBUF; a producer fills it only after the MMAs
+// of tile n - NBUF completed.  Producers may run ahead further than an
+// mbarrier's phase parity can tell apart, so they wait on mma_tiles_done, a
+// monotonic count of completed tiles that the epilogue publishes (release)
+// once all four epilogue warps have read the tile's row destinations.
+// Every wait is bounded; a timeout raises kErrTimeout and the CTA winds down.
+constexpr int kProducerWarps = 27;
+constexpr int kMmaWarp = 27;  // warps 28..31: epilogue
 
 template <int K, int L, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -182,25 +321,40 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               float* __restrict__ partial) {
   static_assert(K % 32 == 0 && K >= 32 && K <= 128, "K must be 32, 64 or 128");
   static_assert(L % 32 == 0 && L >= 32 && L <= 256, "L must be a multiple of 32 in [32, 256]");
-  constexpr int GS = K / 8;            // lanes per row; each lane: two float4 at k0 and k0 + K/2
-  constexpr int GPW = 32 / GS;         // rows per warp pass
-  constexpr int NWARPS = kTcThreads / 32;
+  static_assert(kTcThreads == 1024, "32 warps: 27 producers, 1 MMA, 4 epilogue");
+  using PL = ProdLayout<K>;
+  constexpr int GS = PL::GS, VEC = PL::VEC;
+  static_assert(PL::U <= GS && kQuad <= GS, "one lane per prefetched nonzero and per claimed item");
+  constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
-  constexpr uint32_t NCOLS = L;        // TMEM columns of the fp32 accumulator
+  constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
+  constexpr int TBYTES = kTcRows * K * 4;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ uint64_t mbar;
+  __shared__ uint64_t full_bar[NBUF], mma_bar[NBUF], free_bar[NBUF];
+  __shared__ int2 dest[NBUF][kTcRows];  // per slot: (A row, partial slot); x < 0 = padding
   __shared__ uint32_t tmem_base;
+  __shared__ int claim, fill, fail_flag, mma_tiles_done;
+  __shared__ int last_commit[NBUF];     // last tile committed to each accumulator (-1: none)
   uint8_t* sT = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sD = sT + kTcRows * K * 4;
+  uint8_t* sD = sT + NBUF * TBYTES;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (warp == 0) {
+  if (warp == kMmaWarp) {
     tc::tmem_alloc(&tmem_base, NCOLS);
     tc::tmem_relinquish();
   }
   if (tid == 0) {
-    tc::mbar_init(&mbar, 1);
+    for (int b = 0; b < NBUF; ++b) {
+      tc::mbar_init(&full_bar[b], kTcRows);
+      tc::mbar_init(&mma_bar[b], 1);
+      tc::mbar_init(&free_bar[b], 4);
+      last_commit[b] = -1;
+    }
     tc::fence_mbar_init();
+    claim = 0;
+    fill = 0;
+    fail_flag = 0;
+    mma_tiles_done = 0;
   }
   // D (K x L, row-major) -> D^T as the B operand (L rows of K), tf32
   for (int i = tid; i < K * (L / 4); i += kTcThreads) {
@@ -216,7 +370,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc::tc_fence_after_sync();
   const uint32_t tmem = tmem_base;
-  const uint32_t sT_addr = tc::smem_u32(sT), sD_addr = tc::smem_u32(sD);
 
   int64_t nitems;
   if (MODE == kSegments) {
@@ -226,128 +379,165 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     nitems = dense_rows;
   }
   const int64_t ntiles = (nitems + kTcRows - 1) / kTcRows;
-  const int grp = lane / GS, gl = lane % GS;
-  const int k0 = 4 * gl, k1 = 4 * gl + K / 2;
-  uint32_t phase = 0;
-  bool failed = false;
+  // this CTA's items: rows of item tiles blockIdx.x + j * gridDim.x, j < nlocal
+  const int nlocal = (int)(ntiles > blockIdx.x ? (ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0);
+  int total_rows = nlocal * kTcRows;
+  if (nlocal > 0 && (int64_t)blockIdx.x + (int64_t)(nlocal - 1) * gridDim.x == ntiles - 1)
+    total_rows -= (int)(ntiles * kTcRows - nitems);  // the global last item tile is partial
+  const int pad = nlocal * kTcRows - total_rows;      // padding slots of the last slot tile
 
-  for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
-    // ---- producer: T rows of the tile, tf32, swizzled, in shared memory
-    for (int s = warp * GPW + grp; s < kTcRows; s += NWARPS * GPW) {
-      const int64_t item = t * kTcRows + s;
-      float a[4] = {0.f, 0.f, 0.f, 0.f}, b[4] = {0.f, 0.f, 0.f, 0.f};
-      if (item < nitems) {
-        if (MODE == kSegments) {
-          const int4 sg = __ldg(segs + item);
-          int p = sg.y;
-          const int p1 = sg.z;
-          for (; p + 4 <= p1; p += 4) {
-            int c[4];
-            float v[4];
-            float4 x0[4], x1[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              c[u] = __ldg(crd + p + u);
-              v[u] = __ldg(vals + p + u);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const float* row = X + (int64_t)c[u] * K;
-              x0[u] = __ldg(reinterpret_cast<const float4*>(row + k0));
-              x1[u] = __ldg(reinterpret_cast<const float4*>(row + k1));
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              a[0] = fmaf(v[u], x0[u].x, a[0]); a[1] = fmaf(v[u], x0[u].y, a[1]);
-              a[2] = fmaf(v[u], x0[u].z, a[2]); a[3] = fmaf(v[u], x0[u].w, a[3]);
-              b[0] = fmaf(v[u], x1[u].x, b[0]); b[1] = fmaf(v[u], x1[u].y, b[1]);
-              b[2] = fmaf(v[u], x1[u].z, b[2]); b[3] = fmaf(v[u], x1[u].w, b[3]);
-            }
-          }
-          for (; p < p1; ++p) {
-            const int c = __ldg(crd + p);
-            const float v = __ldg(vals + p);
-            const float* row = X + (int64_t)c * K;
-            const float4 x0 = __ldg(reinterpret_cast<const float4*>(row + k0));
-            const float4 x1 = __ldg(reinterpret_cast<const float4*>(row + k1));
-            a[0] = fmaf(v, x0.x, a[0]); a[1] = fmaf(v, x0.y, a[1]); a[2] = fmaf(v, x0.z, a[2]); a[3] = fmaf(v, x0.w, a[3]);
-            b[0] = fmaf(v, x1.x, b[0]); b[1] = fmaf(v, x1.y, b[1]); b[2] = fmaf(v, x1.z, b[2]); b[3] = fmaf(v, x1.w, b[3]);
-          }
+  if (warp < kProducerWarps) {
+    // ---------------- producers ----------------
+    const int grp = lane / GS, gl = lane % GS, src0 = grp * GS;
+    const unsigned gmask = (GS == 32) ? 0xffffffffu : (((1u << GS) - 1u) << (grp * GS));
+    constexpr int QPT = kTcRows / kQuad;  // claims per item tile
+    // claim c covers local item tile c / QPT, rows (c % QPT) * kQuad + 0..kQuad-1;
+    // lane gl < kQuad of the group loads the record of row gl (x < 0: past the last item)
+    auto load_claim = [&](int c, int4& rec) {
+      rec = make_int4(-1, 0, 0, -1);
+      const int64_t item = ((int64_t)blockIdx.x + (int64_t)(c / QPT) * gridDim.x) * kTcRows + (c % QPT) * kQuad + gl;
+      if (c / QPT < nlocal && gl < kQuad && item < nitems)
+        rec = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
+    };
+    // hands a finished T row of claimed item q to the next free slot
+    int4 rec = make_int4(-1, 0, 0, -1);
+    auto emit = [&](int q, const float4 (&acc)[VEC]) -> bool {
+      const int rx = __shfl_sync(gmask, rec.x, src0 + q), rw = __shfl_sync(gmask, rec.w, src0 + q);
+      if (rx < 0) return true;  // past the last item: no row
+      int slot = 0;
+      if (gl == 0) slot = atomicAdd(&fill, 1);
+      slot = __shfl_sync(gmask, slot, src0);
+      const int n = slot / kTcRows, s = slot % kTcRows, b = n % NBUF;
+      if (n >= NBUF) {  // buffer b is free once the MMAs of slot tile n - NBUF completed
+        const bool ok = count_wait_timeout(&mma_tiles_done, n - NBUF + 1);
+        if (!__all_sync(gmask, ok)) return false;
+      }
+      store_t_row<VEC>(sT + b * TBYTES, s, gl, K, acc);
+      if (gl == 0) dest[b][s] = make_int2(rx, rw);
+      tc::fence_proxy_async_smem();
+      __syncwarp(gmask);
+      if (gl == 0) {
+        if (slot == total_rows - 1 && pad > 0) {  // the last row: pad the final slot tile
+          for (int i = s + 1; i < kTcRows; ++i) dest[b][i] = make_int2(-1, -1);
+          tc::mbar_arrive_n(&full_bar[b], 1 + pad);
         } else {
-          const float* row = X + item * K;
-          const float4 x0 = __ldg(reinterpret_cast<const float4*>(row + k0));
-          const float4 x1 = __ldg(reinterpret_cast<const float4*>(row + k1));
-          a[0] = x0.x; a[1] = x0.y; a[2] = x0.z; a[3] = x0.w;
-          b[0] = x1.x; b[1] = x1.y; b[2] = x1.z; b[3] = x1.w;
+          tc::mbar_arrive(&full_bar[b]);
         }
       }
-      *reinterpret_cast<uint4*>(sT + tc::sw128_offset(s, k0, kTcRows)) =
-          make_uint4(tc::to_tf32(a[0]), tc::to_tf32(a[1]), tc::to_tf32(a[2]), tc::to_tf32(a[3]));
-      *reinterpret_cast<uint4*>(sT + tc::sw128_offset(s, k1, kTcRows)) =
-          make_uint4(tc::to_tf32(b[0]), tc::to_tf32(b[1]), tc::to_tf32(b[2]), tc::to_tf32(b[3]));
+      return true;
+    };
+    int cl = 0, x = 0;
+    if (gl == 0) x = atomicAdd(&claim, 1);
+    cl = __shfl_sync(gmask, x, src0);
+    load_claim(cl, rec);
+    while (cl / QPT < nlocal) {
+      x = 0;
+      if (gl == 0) x = atomicAdd(&claim, 1);
+      const int cl_next = __shfl_sync(gmask, x, src0);
+      int4 rec_next;
+      load_claim(cl_next, rec_next);  // loads while this claim is built
+      bool ok = true;
+      if (MODE == kSegments) {
+        // items past the last one get an empty range at the end of the last valid item
+        const unsigned valid = (__ballot_sync(gmask, gl < kQuad && rec.x >= 0) >> src0) & ((1u << kQuad) - 1u);
+        const int nvalid = __popc(valid);
+        const int start0 = __shfl_sync(gmask, rec.y, src0);
+        const int last_end = __shfl_sync(gmask, rec.z, src0 + (nvalid > 0 ? nvalid - 1 : 0));
+        const int my_end = rec.x >= 0 ? rec.z : (nvalid > 0 ? last_end : start0);
+        ok = build_quad<K, VEC, PL::U>(my_end, nvalid > 0 ? start0 : 0, gmask, src0, gl, crd, vals, X, emit);
+      } else {
+#pragma unroll
+        for (int q = 0; q < kQuad && ok; ++q) {
+          const int rx = __shfl_sync(gmask, rec.x, src0 + q);
+          float4 acc[VEC];
+#pragma unroll
+          for (int w = 0; w < VEC; ++w)
+            acc[w] = rx >= 0 ? __ldg(reinterpret_cast<const float4*>(X + (int64_t)rx * K + 4 * gl + w * (K / VEC)))
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+          ok = emit(q, acc);
+        }
+      }
+      if (!ok) {
+        atomicOr(&fail_flag, 1);
+        break;
+      }
+      cl = cl_next;
+      rec = rec_next;
     }
-    tc::fence_proxy_async_smem();
-    tc::tc_fence_before_sync();
-    __syncthreads();
-    // ---- MMA: one thread issues the tile's K/8 steps, then commits to mbar
-    if (tid == 0) {
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t sT_addr = tc::smem_u32(sT), sD_addr = tc::smem_u32(sD);
+      for (int j = 0; j < nlocal; ++j) {
+        const int b = j % NBUF;
+        if (!mbar_wait_timeout(&full_bar[b], (j / NBUF) & 1) ||
+            (j >= NBUF && !mbar_wait_timeout(&free_bar[b], ((j / NBUF) - 1) & 1))) {
+          atomicOr(&fail_flag, 1);
+          break;
+        }
+        tc::tc_fence_after_sync();
+        const uint32_t a_base = sT_addr + b * TBYTES;
+#pragma unroll
+        for (int kb = 0; kb < K / 32; ++kb)
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t ad = tc::desc_k_sw128(a_base + kb * kTcRows * 128 + ks * 32);
+            const uint64_t bd = tc::desc_k_sw128(sD_addr + kb * L * 128 + ks * 32);
+            tc::mma_tf32(tmem + (uint32_t)(b * L), ad, bd, IDESC, (kb | ks) != 0);
+          }
+        tc::mma_commit(&mma_bar[b]);
+        last_commit[b] = j;
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;  // TMEM lane quadrant of this warp
+    for (int j = 0; j < nlocal; ++j) {
+      const int b = j % NBUF;
+      const bool ok = mbar_wait_timeout(&mma_bar[b], (j / NBUF) & 1);
+      if (!__all_sync(0xffffffffu, ok)) {
+        atomicOr(&fail_flag, 1);
+        break;
+      }
       tc::tc_fence_after_sync();
-#pragma unroll
-      for (int kb = 0; kb < K / 32; ++kb)
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-          const uint64_t ad = tc::desc_k_sw128(sT_addr + kb * kTcRows * 128 + ks * 32);
-          const uint64_t bd = tc::desc_k_sw128(sD_addr + kb * L * 128 + ks * 32);
-          tc::mma_tf32(tmem, ad, bd, IDESC, (kb | ks) != 0);
-        }
-      tc::mma_commit(&mbar);
-    }
-    const bool ok = mbar_wait_timeout(&mbar, phase);
-    phase ^= 1u;
-    if (__syncthreads_or(!ok)) {
-      failed = true;
-      break;
-    }
-    tc::tc_fence_after_sync();
-    // ---- epilogue: warp w reads TMEM lanes 32*(w%4).., columns slice w/4
-    {
-      const int q = warp & 3, j = warp >> 2;
       const int rr = 32 * q + lane;
-      const int64_t item = t * kTcRows + rr;
+      const int2 dd = dest[b][rr];
+      // all four epilogue warps have their destinations: the slot tile may be refilled
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (q == 0 && lane == 0) tc::st_release_smem(&mma_tiles_done, j + 1);
       float* dst = nullptr;
-      if (item < nitems) {
-        if (MODE == kSegments) {
-          const int4 sg = __ldg(segs + item);
-          dst = sg.w < 0 ? A + (int64_t)sg.x * L : partial + (int64_t)sg.w * L;
-        } else {
-          dst = A + item * L;
-        }
-      }
-      constexpr int CW = L / 4;  // columns per warp
-#pragma unroll
-      for (int c = 0; c < CW; c += 8) {
+      if (dd.x >= 0) dst = dd.y < 0 ? A + (int64_t)dd.x * L : partial + (int64_t)dd.y * L;
+#pragma unroll 4
+      for (int c = 0; c < L; c += 8) {
         float v[8];
-        tc::tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(j * CW + c), v);
+        tc::tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
         if (dst != nullptr) {
-          float4* o = reinterpret_cast<float4*>(dst + j * CW + c);
+          float4* o = reinterpret_cast<float4*>(dst + c);
           o[0] = make_float4(v[0], v[1], v[2], v[3]);
           o[1] = make_float4(v[4], v[5], v[6], v[7]);
         }
       }
+      tc::tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&free_bar[b]);
     }
-    tc::tc_fence_before_sync();
-    __syncthreads();
   }
-  if (failed) {
-    // the MMAs of the abandoned tile may still be running: wait once more
-    // (bounded) before the tensor memory is released
-    mbar_wait_timeout(&mbar, phase ^ 1u);
-    if (tid == 0) atomicOr(&hdr->error, kErrTimeout);
-  }
+
+  // ---- teardown: every role has finished its loop
   tc::tc_fence_before_sync();
   __syncthreads();
+  if (fail_flag) {
+    // MMAs of abandoned tiles may still be running: wait (bounded) for each
+    // accumulator's last commit before the tensor memory is released
+    if (warp == kMmaWarp && lane == 0)
+      for (int b = 0; b < NBUF; ++b)
+        if (last_commit[b] >= 0) mbar_wait_timeout(&mma_bar[b], (last_commit[b] / NBUF) & 1);
+    if (tid == 0) atomicOr(&hdr->error, kErrTimeout);
+  }
+  __syncthreads();
   tc::tc_fence_after_sync();
-  if (warp == 0) tc::tmem_dealloc(tmem, NCOLS);
+  if (warp == kMmaWarp) tc::tmem_dealloc(tmem, NCOLS);
 }
 
 struct TcLaunch {
@@ -369,12 +559,16 @@ cudaError_t tc_setup(TcLaunch* out) {
   if ((e = cudaDeviceGetAttribute(&sm_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
   size_t smem = tc_smem_bytes(K, L);
-  // no more resident CTAs per SM than tensor memory holds accumulators for
-  const int max_ctas = 512 / L;
+  // no more resident CTAs per SM than tensor memory (512 columns) holds
+  // accumulators for: a CTA waiting in tcgen05.alloc would only idle
+  const int max_ctas = 512 / (tc_nbuf(K, L) * L);
   const size_t floor_bytes = (size_t)sm_smem / (size_t)(max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
   if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
       cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                (int)cudaSharedmemCarveoutMaxShared)) != cudaSuccess)
     return e;
   int occ = 0;
   if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_tc_gemm<K, L, MODE>, kTcThreads, smem)) !=
@@ -407,7 +601,7 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
   }
   SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
   SLNR_TC_CASE(64, 32) SLNR_TC_CASE(64, 64) SLNR_TC_CASE(64, 128) SLNR_TC_CASE(64, 256)
-  SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128) SLNR_TC_CASE(128, 256)
+  SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128)
 #undef SLNR_TC_CASE
   return cudaErrorInvalidValue;
 }
@@ -415,7 +609,8 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
 }  // namespace
 
 bool tc_supported(int K, int L) {
-  return (K == 32 || K == 64 || K == 128) && (L == 32 || L == 64 || L == 128 || L == 256);
+  return (K == 32 || K == 64 || K == 128) && (L == 32 || L == 64 || L == 128 || L == 256) &&
+         tc_smem_bytes(K, L) <= (size_t)200 * 1024;
 }
 
 int seg_scan_blocks(int64_t nrows) { return (int)((nrows + kScanRows - 1) / kScanRows); }

@@ -50,6 +50,7 @@ def test_full_size_sampled(slnr, idx):
     B, dense = P.to_device(w)
     out = slnr.run(w.op, B, dense, variant="fused", allow_tf32=True)
     torch.cuda.synchronize()
+    assert slnr.device_flags() == 0, f"device flags {slnr.device_flags():#x}"
     rows = sample_rows(w)
     ref, ref_abs = oracle.get().run(w, rows=rows)
     got = P.values_of(w.op, out)[torch.from_numpy(rows).long().cuda()].cpu().numpy()
