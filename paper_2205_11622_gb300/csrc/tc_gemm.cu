@@ -162,8 +162,10 @@ __global__ void __launch_bounds__(kScanThreads) k_seg_write(int nrows, const int
 // Waits until *count >= target (a monotonic shared-memory counter); false on timeout.
 __device__ __forceinline__ bool count_wait_timeout(const int* count, int target) {
   const long long t0 = clock64();
-  while (tc::ld_acquire_smem(count) < target)
+  while (tc::ld_acquire_smem(count) < target) {
+    __nanosleep(64);  // leave the issue slots to the warps that are working
     if (clock64() - t0 > kWaitCycles) return false;
+  }
   return true;
 }
 
@@ -188,107 +190,127 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
   return (size_t)tc_nbuf(K, L) * kTcRows * K * 4 + (size_t)L * K * 4 + 1024;
 }
 
-#ifndef SLNR_TC_VEC_K128
-#define SLNR_TC_VEC_K128 1  // float4 per lane, K = 128
+#ifndef SLNR_TC_ROWS_IN_FLIGHT
+#define SLNR_TC_ROWS_IN_FLIGHT 8  // gathered rows of X in flight per producer warp (K <= 64)
 #endif
-#ifndef SLNR_TC_U_K128
-#define SLNR_TC_U_K128 4    // rows in flight per group, K = 128
-#endif
-#ifndef SLNR_TC_VEC_K64
-#define SLNR_TC_VEC_K64 1   // float4 per lane, K <= 64
-#endif
-#ifndef SLNR_TC_U_K64
-#define SLNR_TC_U_K64 4     // rows in flight per group, K <= 64
+#ifndef SLNR_TC_ROWS_IN_FLIGHT_K128
+#define SLNR_TC_ROWS_IN_FLIGHT_K128 4  // the same for K = 128 (register budget)
 #endif
 
-// Lane layout of the producer: a group of GS lanes builds T rows; lane gl
-// holds VEC float4 of a row, at columns 4*gl + v*(K/VEC) (v < VEC), and
-// keeps U gathered rows of X in flight.  A claim is kQuad consecutive items
-// (segments), whose nonzeros form one contiguous range.
+// Producer layout: a whole warp builds one T row at a time (no divergence
+// inside a warp); lane l holds the F = K/32 consecutive values
+// [F*l, F*l + F), loaded as one float / float2 / float4, so each gathered
+// row is one coalesced warp load.  U rows are in flight per warp (build-time
+// defaults below).  A claim is
+// kQuad consecutive items (segments), whose nonzeros form one contiguous
+// range.
 template <int K>
 struct ProdLayout {
-  static constexpr int VEC = K >= 128 ? SLNR_TC_VEC_K128 : SLNR_TC_VEC_K64;
-  static constexpr int GS = K / (4 * VEC);
-  static constexpr int U = K >= 128 ? SLNR_TC_U_K128 : SLNR_TC_U_K64;
+  static constexpr int F = K / 32;
+  static constexpr int U = K >= 128 ? SLNR_TC_ROWS_IN_FLIGHT_K128 : SLNR_TC_ROWS_IN_FLIGHT;
 };
 constexpr int kQuad = 4;
 
-template <int VEC>
-__device__ __forceinline__ void store_t_row(uint8_t* sTb, int s, int gl, int K, const float4 (&acc)[VEC]) {
+template <int F>
+struct Frag {
+  float v[F];
+};
+
+template <int F>
+__device__ __forceinline__ Frag<F> ldg_frag(const float* __restrict__ p) {
+  Frag<F> r;
+  if constexpr (F == 4) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(p));
+    r.v[0] = a.x; r.v[1] = a.y; r.v[2] = a.z; r.v[3] = a.w;
+  } else if constexpr (F == 2) {
+    const float2 a = __ldg(reinterpret_cast<const float2*>(p));
+    r.v[0] = a.x; r.v[1] = a.y;
+  } else {
+    r.v[0] = __ldg(p);
+  }
+  return r;
+}
+
+template <int F>
+__device__ __forceinline__ Frag<F> zero_frag() {
+  Frag<F> r;
 #pragma unroll
-  for (int w = 0; w < VEC; ++w)
-    *reinterpret_cast<uint4*>(sTb + tc::sw128_offset(s, 4 * gl + w * (K / VEC), kTcRows)) =
-        make_uint4(tc::to_tf32(acc[w].x), tc::to_tf32(acc[w].y), tc::to_tf32(acc[w].z), tc::to_tf32(acc[w].w));
+  for (int e = 0; e < F; ++e) r.v[e] = 0.f;
+  return r;
+}
+
+// T row s of buffer sTb, lane's values [F*lane, F*lane+F), rounded to tf32.
+template <int K>
+__device__ __forceinline__ void store_t_row(uint8_t* sTb, int s, int lane, const Frag<K / 32>& acc) {
+  constexpr int F = K / 32;
+  uint8_t* dst = sTb + tc::sw128_offset(s, F * lane, kTcRows);
+  if constexpr (F == 4) {
+    *reinterpret_cast<uint4*>(dst) =
+        make_uint4(tc::to_tf32(acc.v[0]), tc::to_tf32(acc.v[1]), tc::to_tf32(acc.v[2]), tc::to_tf32(acc.v[3]));
+  } else if constexpr (F == 2) {
+    *reinterpret_cast<uint2*>(dst) = make_uint2(tc::to_tf32(acc.v[0]), tc::to_tf32(acc.v[1]));
+  } else {
+    *reinterpret_cast<uint32_t*>(dst) = tc::to_tf32(acc.v[0]);
+  }
 }
 
 // Accumulates the kQuad rows of one claim: row q sums vals[p] X[crd[p],:] over
-// its range, which ends at the value lane src0+q of the group holds in my_end;
-// the ranges are consecutive from p, so one pipeline of U row gathers runs
-// over all of them, and emit(q, acc) hands each row on as soon as its range is
-// done (returns false to abandon the claim).  Coordinates and values of the
-// next batch are fetched while the current rows are in flight, each by one
-// lane of the group and passed on by shuffles.
-template <int K, int VEC, int U, typename Emit>
-__device__ __forceinline__ bool build_quad(int my_end, int p, unsigned gmask, int src0, int gl,
-                                           const int32_t* __restrict__ crd, const float* __restrict__ vals,
-                                           const float* __restrict__ X, Emit&& emit) {
-  const int p_end = __shfl_sync(gmask, my_end, src0 + kQuad - 1);
-  float4 acc[VEC];
-#pragma unroll
-  for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+// its range, which ends at the value lane q holds in my_end; the ranges are
+// consecutive from p, so one pipeline of U row gathers runs over all of them,
+// and emit(q, acc) hands each row on as soon as its range is done (returns
+// false to abandon the claim).  Coordinates and values of the next batch are
+// fetched while the current rows are in flight, one nonzero per lane, and
+// passed on by shuffles.
+template <int K, int U, typename Emit>
+__device__ __forceinline__ bool build_quad(int my_end, int p, int lane, const int32_t* __restrict__ crd,
+                                           const float* __restrict__ vals, const float* __restrict__ X,
+                                           Emit&& emit) {
+  constexpr int F = K / 32;
+  static_assert(U <= 32 && kQuad <= 32, "one lane per prefetched nonzero and per row");
+  const int p_end = __shfl_sync(0xffffffffu, my_end, kQuad - 1);
+  Frag<F> acc = zero_frag<F>();
   int q = 0;
-  int cur_end = __shfl_sync(gmask, my_end, src0);
+  int cur_end = __shfl_sync(0xffffffffu, my_end, 0);
   int my_c = 0;
   float my_v = 0.f;
-  if (gl < U && p + gl < p_end) {
-    my_c = __ldg(crd + p + gl);
-    my_v = __ldg(vals + p + gl);
+  if (lane < U && p + lane < p_end) {
+    my_c = __ldg(crd + p + lane);
+    my_v = __ldg(vals + p + lane);
   }
   while (p < p_end) {
     float v[U];
-    float4 x[U][VEC];
+    Frag<F> x[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int cu = __shfl_sync(gmask, my_c, src0 + u);
-      v[u] = __shfl_sync(gmask, my_v, src0 + u);
-      const float* row = X + (int64_t)cu * K + 4 * gl;
-#pragma unroll
-      for (int w = 0; w < VEC; ++w)
-        x[u][w] = (p + u < p_end) ? __ldg(reinterpret_cast<const float4*>(row + w * (K / VEC)))
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int cu = __shfl_sync(0xffffffffu, my_c, u);
+      v[u] = __shfl_sync(0xffffffffu, my_v, u);
+      x[u] = (p + u < p_end) ? ldg_frag<F>(X + (int64_t)cu * K + F * lane) : zero_frag<F>();
     }
     const int pn = p + U;
     my_c = 0;
     my_v = 0.f;
-    if (gl < U && pn + gl < p_end) {
-      my_c = __ldg(crd + pn + gl);
-      my_v = __ldg(vals + pn + gl);
+    if (lane < U && pn + lane < p_end) {
+      my_c = __ldg(crd + pn + lane);
+      my_v = __ldg(vals + pn + lane);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (p + u < p_end) {
         while (p + u >= cur_end) {  // rows whose range is complete (empty rows included)
           if (!emit(q, acc)) return false;
-#pragma unroll
-          for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+          acc = zero_frag<F>();
           ++q;
-          cur_end = __shfl_sync(gmask, my_end, src0 + q);
+          cur_end = __shfl_sync(0xffffffffu, my_end, q);
         }
 #pragma unroll
-        for (int w = 0; w < VEC; ++w) {
-          acc[w].x = fmaf(v[u], x[u][w].x, acc[w].x);
-          acc[w].y = fmaf(v[u], x[u][w].y, acc[w].y);
-          acc[w].z = fmaf(v[u], x[u][w].z, acc[w].z);
-          acc[w].w = fmaf(v[u], x[u][w].w, acc[w].w);
-        }
+        for (int e = 0; e < F; ++e) acc.v[e] = fmaf(v[u], x[u].v[e], acc.v[e]);
       }
     }
     p = pn;
   }
   for (; q < kQuad; ++q) {
     if (!emit(q, acc)) return false;
-#pragma unroll
-    for (int w = 0; w < VEC; ++w) acc[w] = make_float4(0.f, 0.f, 0.f, 0.f);
+    acc = zero_frag<F>();
   }
   return true;
 }
@@ -323,8 +345,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   static_assert(L % 32 == 0 && L >= 32 && L <= 256, "L must be a multiple of 32 in [32, 256]");
   static_assert(kTcThreads == 1024, "32 warps: 27 producers, 1 MMA, 4 epilogue");
   using PL = ProdLayout<K>;
-  constexpr int GS = PL::GS, VEC = PL::VEC;
-  static_assert(PL::U <= GS && kQuad <= GS, "one lane per prefetched nonzero and per claimed item");
+  constexpr int F = PL::F;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
   constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
@@ -388,35 +409,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (warp < kProducerWarps) {
     // ---------------- producers ----------------
-    const int grp = lane / GS, gl = lane % GS, src0 = grp * GS;
-    const unsigned gmask = (GS == 32) ? 0xffffffffu : (((1u << GS) - 1u) << (grp * GS));
     constexpr int QPT = kTcRows / kQuad;  // claims per item tile
     // claim c covers local item tile c / QPT, rows (c % QPT) * kQuad + 0..kQuad-1;
-    // lane gl < kQuad of the group loads the record of row gl (x < 0: past the last item)
+    // lane q < kQuad loads the record of row q (x < 0: past the last item)
     auto load_claim = [&](int c, int4& rec) {
       rec = make_int4(-1, 0, 0, -1);
-      const int64_t item = ((int64_t)blockIdx.x + (int64_t)(c / QPT) * gridDim.x) * kTcRows + (c % QPT) * kQuad + gl;
-      if (c / QPT < nlocal && gl < kQuad && item < nitems)
+      const int64_t item =
+          ((int64_t)blockIdx.x + (int64_t)(c / QPT) * gridDim.x) * kTcRows + (c % QPT) * kQuad + lane;
+      if (c / QPT < nlocal && lane < kQuad && item < nitems)
         rec = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
     };
     // hands a finished T row of claimed item q to the next free slot
     int4 rec = make_int4(-1, 0, 0, -1);
-    auto emit = [&](int q, const float4 (&acc)[VEC]) -> bool {
-      const int rx = __shfl_sync(gmask, rec.x, src0 + q), rw = __shfl_sync(gmask, rec.w, src0 + q);
+    auto emit = [&](int q, const Frag<F>& acc) -> bool {
+      const int rx = __shfl_sync(0xffffffffu, rec.x, q), rw = __shfl_sync(0xffffffffu, rec.w, q);
       if (rx < 0) return true;  // past the last item: no row
       int slot = 0;
-      if (gl == 0) slot = atomicAdd(&fill, 1);
-      slot = __shfl_sync(gmask, slot, src0);
+      if (lane == 0) slot = atomicAdd(&fill, 1);
+      slot = __shfl_sync(0xffffffffu, slot, 0);
       const int n = slot / kTcRows, s = slot % kTcRows, b = n % NBUF;
       if (n >= NBUF) {  // buffer b is free once the MMAs of slot tile n - NBUF completed
         const bool ok = count_wait_timeout(&mma_tiles_done, n - NBUF + 1);
-        if (!__all_sync(gmask, ok)) return false;
+        if (!__all_sync(0xffffffffu, ok)) return false;
       }
-      store_t_row<VEC>(sT + b * TBYTES, s, gl, K, acc);
-      if (gl == 0) dest[b][s] = make_int2(rx, rw);
+      store_t_row<K>(sT + b * TBYTES, s, lane, acc);
+      if (lane == 0) dest[b][s] = make_int2(rx, rw);
       tc::fence_proxy_async_smem();
-      __syncwarp(gmask);
-      if (gl == 0) {
+      __syncwarp();
+      if (lane == 0) {
         if (slot == total_rows - 1 && pad > 0) {  // the last row: pad the final slot tile
           for (int i = s + 1; i < kTcRows; ++i) dest[b][i] = make_int2(-1, -1);
           tc::mbar_arrive_n(&full_bar[b], 1 + pad);
@@ -426,34 +446,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       return true;
     };
-    int cl = 0, x = 0;
-    if (gl == 0) x = atomicAdd(&claim, 1);
-    cl = __shfl_sync(gmask, x, src0);
+    int x = 0;
+    if (lane == 0) x = atomicAdd(&claim, 1);
+    int cl = __shfl_sync(0xffffffffu, x, 0);
     load_claim(cl, rec);
     while (cl / QPT < nlocal) {
       x = 0;
-      if (gl == 0) x = atomicAdd(&claim, 1);
-      const int cl_next = __shfl_sync(gmask, x, src0);
+      if (lane == 0) x = atomicAdd(&claim, 1);
+      const int cl_next = __shfl_sync(0xffffffffu, x, 0);
       int4 rec_next;
       load_claim(cl_next, rec_next);  // loads while this claim is built
       bool ok = true;
       if (MODE == kSegments) {
         // items past the last one get an empty range at the end of the last valid item
-        const unsigned valid = (__ballot_sync(gmask, gl < kQuad && rec.x >= 0) >> src0) & ((1u << kQuad) - 1u);
+        const unsigned valid = __ballot_sync(0xffffffffu, lane < kQuad && rec.x >= 0) & ((1u << kQuad) - 1u);
         const int nvalid = __popc(valid);
-        const int start0 = __shfl_sync(gmask, rec.y, src0);
-        const int last_end = __shfl_sync(gmask, rec.z, src0 + (nvalid > 0 ? nvalid - 1 : 0));
+        const int start0 = __shfl_sync(0xffffffffu, rec.y, 0);
+        const int last_end = __shfl_sync(0xffffffffu, rec.z, nvalid > 0 ? nvalid - 1 : 0);
         const int my_end = rec.x >= 0 ? rec.z : (nvalid > 0 ? last_end : start0);
-        ok = build_quad<K, VEC, PL::U>(my_end, nvalid > 0 ? start0 : 0, gmask, src0, gl, crd, vals, X, emit);
+        ok = build_quad<K, PL::U>(my_end, nvalid > 0 ? start0 : 0, lane, crd, vals, X, emit);
       } else {
 #pragma unroll
         for (int q = 0; q < kQuad && ok; ++q) {
-          const int rx = __shfl_sync(gmask, rec.x, src0 + q);
-          float4 acc[VEC];
-#pragma unroll
-          for (int w = 0; w < VEC; ++w)
-            acc[w] = rx >= 0 ? __ldg(reinterpret_cast<const float4*>(X + (int64_t)rx * K + 4 * gl + w * (K / VEC)))
-                             : make_float4(0.f, 0.f, 0.f, 0.f);
+          const int rx = __shfl_sync(0xffffffffu, rec.x, q);
+          const Frag<F> acc = rx >= 0 ? ldg_frag<F>(X + (int64_t)rx * K + F * lane) : zero_frag<F>();
           ok = emit(q, acc);
         }
       }
@@ -508,14 +524,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (q == 0 && lane == 0) tc::st_release_smem(&mma_tiles_done, j + 1);
       float* dst = nullptr;
       if (dd.x >= 0) dst = dd.y < 0 ? A + (int64_t)dd.x * L : partial + (int64_t)dd.y * L;
-#pragma unroll 4
-      for (int c = 0; c < L; c += 8) {
-        float v[8];
-        tc::tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
+#pragma unroll 1
+      for (int c = 0; c < L; c += 32) {
+        float v[32];
+        tc::tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
         if (dst != nullptr) {
           float4* o = reinterpret_cast<float4*>(dst + c);
-          o[0] = make_float4(v[0], v[1], v[2], v[3]);
-          o[1] = make_float4(v[4], v[5], v[6], v[7]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
       }
       tc::tc_fence_before_sync();
