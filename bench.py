@@ -235,6 +235,22 @@ def dist_env():
     return rank, world, local
 
 
+def job_throughput(step_ms, step_flops, world, pg=None, device=None):
+    """Whole-job throughput of replicas: every rank runs the same step on its
+    own GPU, the job takes as long as the slowest rank (max over ranks of the
+    step time), and the job does world x step_flops of useful work in that
+    time.  Returns (max step ms, GFLOP/s).  pg is torch.distributed (or None
+    for one process); device is where the reduction tensor lives (a CUDA
+    device under NCCL, the CPU under gloo)."""
+    if pg is not None:
+        import torch
+        t = torch.tensor([float(step_ms)], dtype=torch.float64, device=device)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        step_ms = float(t.item())
+        pg.barrier()
+    return step_ms, world * step_flops / (step_ms / 1e3) / 1e9
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
@@ -392,14 +408,8 @@ def main():
     time.sleep(0.3)
     clocks.stop()
     mean_ms = [statistics.mean(x) for x in expr_ms]
-    step_ms = sum(mean_ms)
-    if pg is not None:
-        t = torch.tensor([step_ms], dtype=torch.float64, device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        step_ms = float(t.item())
-        pg.barrier()
     total_flops = sum(flops)
-    value = world * total_flops / (step_ms / 1e3) / 1e9
+    step_ms, value = job_throughput(sum(mean_ms), total_flops, world, pg, dev)
 
     peak, peak_kind = measured_peaks()
     per_expression = {}

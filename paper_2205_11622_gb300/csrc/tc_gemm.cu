@@ -6,7 +6,7 @@
 // chip and A(r,:) = T(r,:) . D follows at once.  Rows are grouped into
 // "segments" of at most kSegChunk nonzeros (a row with more nonzeros becomes
 // several chunk segments); a persistent CTA takes 128 segments at a time:
-//   producer: 16 warps gather C rows into registers and write the 128 x K
+//   producer: 27 warps gather C rows into registers and write the 128 x K
 //             tile of T, rounded to tf32, into shared memory (128B-swizzled,
 //             K-major) -- T never goes to global memory;
 //   MMA:      one thread issues K/8 tcgen05.mma (M=128, N=L, K=8) with D^T,
@@ -190,148 +190,58 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
   return (size_t)tc_nbuf(K, L) * kTcRows * K * 4 + (size_t)L * K * 4 + 1024;
 }
 
-#ifndef SLNR_TC_ROWS_IN_FLIGHT
-#define SLNR_TC_ROWS_IN_FLIGHT 8  // gathered rows of X in flight per producer warp (K <= 64)
+#ifndef SLNR_TC_VPL
+#define SLNR_TC_VPL 4  // T-row columns per producer lane (4 or 8)
 #endif
-#ifndef SLNR_TC_ROWS_IN_FLIGHT_K128
-#define SLNR_TC_ROWS_IN_FLIGHT_K128 4  // the same for K = 128 (register budget)
+#ifndef SLNR_TC_UNROLL
+#define SLNR_TC_UNROLL 8  // gathered rows in flight per lane group
 #endif
 
-// Producer layout: a whole warp builds one T row at a time (no divergence
-// inside a warp); lane l holds the F = K/32 consecutive values
-// [F*l, F*l + F), loaded as one float / float2 / float4, so each gathered
-// row is one coalesced warp load.  U rows are in flight per warp (build-time
-// defaults below).  A claim is
-// kQuad consecutive items (segments), whose nonzeros form one contiguous
-// range.
+// Producer layout: a T row is built by a group of GS = K / VPL lanes, lane gl
+// of the group holding the VPL columns [VPL*gl, VPL*gl + VPL), loaded as
+// float4s; a warp builds G = 32 / GS rows at once, one per group, with U row
+// gathers in flight per group.  A claim is the G consecutive items of one
+// warp pass.
 template <int K>
 struct ProdLayout {
-  static constexpr int F = K / 32;
-  static constexpr int U = K >= 128 ? SLNR_TC_ROWS_IN_FLIGHT_K128 : SLNR_TC_ROWS_IN_FLIGHT;
-};
-constexpr int kQuad = 4;
-
-template <int F>
-struct Frag {
-  float v[F];
+  static constexpr int VPL = K / SLNR_TC_VPL >= 1 && K / SLNR_TC_VPL <= 32 ? SLNR_TC_VPL : 4;
+  static constexpr int GS = K / VPL;
+  static constexpr int G = 32 / GS;
+  static constexpr int U = SLNR_TC_UNROLL;
+  static_assert(VPL == 4 || VPL == 8, "VPL must be 4 or 8");
+  static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
 };
 
-template <int F>
-__device__ __forceinline__ Frag<F> ldg_frag(const float* __restrict__ p) {
-  Frag<F> r;
-  if constexpr (F == 4) {
-    const float4 a = __ldg(reinterpret_cast<const float4*>(p));
-    r.v[0] = a.x; r.v[1] = a.y; r.v[2] = a.z; r.v[3] = a.w;
-  } else if constexpr (F == 2) {
-    const float2 a = __ldg(reinterpret_cast<const float2*>(p));
-    r.v[0] = a.x; r.v[1] = a.y;
-  } else {
-    r.v[0] = __ldg(p);
-  }
-  return r;
-}
-
-template <int F>
-__device__ __forceinline__ Frag<F> zero_frag() {
-  Frag<F> r;
+// Stores the VPL values of lane group column col of T row s (buffer sTb),
+// rounded to tf32, into the 128B-swizzled K-major tile.
+template <int VPL>
+__device__ __forceinline__ void store_t_part(uint8_t* sTb, int s, int col, const float (&acc)[VPL]) {
 #pragma unroll
-  for (int e = 0; e < F; ++e) r.v[e] = 0.f;
-  return r;
-}
-
-// T row s of buffer sTb, lane's values [F*lane, F*lane+F), rounded to tf32.
-template <int K>
-__device__ __forceinline__ void store_t_row(uint8_t* sTb, int s, int lane, const Frag<K / 32>& acc) {
-  constexpr int F = K / 32;
-  uint8_t* dst = sTb + tc::sw128_offset(s, F * lane, kTcRows);
-  if constexpr (F == 4) {
-    *reinterpret_cast<uint4*>(dst) =
-        make_uint4(tc::to_tf32(acc.v[0]), tc::to_tf32(acc.v[1]), tc::to_tf32(acc.v[2]), tc::to_tf32(acc.v[3]));
-  } else if constexpr (F == 2) {
-    *reinterpret_cast<uint2*>(dst) = make_uint2(tc::to_tf32(acc.v[0]), tc::to_tf32(acc.v[1]));
-  } else {
-    *reinterpret_cast<uint32_t*>(dst) = tc::to_tf32(acc.v[0]);
-  }
-}
-
-// Accumulates the kQuad rows of one claim: row q sums vals[p] X[crd[p],:] over
-// its range, which ends at the value lane q holds in my_end; the ranges are
-// consecutive from p, so one pipeline of U row gathers runs over all of them,
-// and emit(q, acc) hands each row on as soon as its range is done (returns
-// false to abandon the claim).  Coordinates and values of the next batch are
-// fetched while the current rows are in flight, one nonzero per lane, and
-// passed on by shuffles.
-template <int K, int U, typename Emit>
-__device__ __forceinline__ bool build_quad(int my_end, int p, int lane, const int32_t* __restrict__ crd,
-                                           const float* __restrict__ vals, const float* __restrict__ X,
-                                           Emit&& emit) {
-  constexpr int F = K / 32;
-  static_assert(U <= 32 && kQuad <= 32, "one lane per prefetched nonzero and per row");
-  const int p_end = __shfl_sync(0xffffffffu, my_end, kQuad - 1);
-  Frag<F> acc = zero_frag<F>();
-  int q = 0;
-  int cur_end = __shfl_sync(0xffffffffu, my_end, 0);
-  int my_c = 0;
-  float my_v = 0.f;
-  if (lane < U && p + lane < p_end) {
-    my_c = __ldg(crd + p + lane);
-    my_v = __ldg(vals + p + lane);
-  }
-  while (p < p_end) {
-    float v[U];
-    Frag<F> x[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int cu = __shfl_sync(0xffffffffu, my_c, u);
-      v[u] = __shfl_sync(0xffffffffu, my_v, u);
-      x[u] = (p + u < p_end) ? ldg_frag<F>(X + (int64_t)cu * K + F * lane) : zero_frag<F>();
-    }
-    const int pn = p + U;
-    my_c = 0;
-    my_v = 0.f;
-    if (lane < U && pn + lane < p_end) {
-      my_c = __ldg(crd + pn + lane);
-      my_v = __ldg(vals + pn + lane);
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (p + u < p_end) {
-        while (p + u >= cur_end) {  // rows whose range is complete (empty rows included)
-          if (!emit(q, acc)) return false;
-          acc = zero_frag<F>();
-          ++q;
-          cur_end = __shfl_sync(0xffffffffu, my_end, q);
-        }
-#pragma unroll
-        for (int e = 0; e < F; ++e) acc.v[e] = fmaf(v[u], x[u].v[e], acc.v[e]);
-      }
-    }
-    p = pn;
-  }
-  for (; q < kQuad; ++q) {
-    if (!emit(q, acc)) return false;
-    acc = zero_frag<F>();
-  }
-  return true;
+  for (int h = 0; h < VPL / 4; ++h)
+    *reinterpret_cast<uint4*>(sTb + tc::sw128_offset(s, col + 4 * h, kTcRows)) =
+        make_uint4(tc::to_tf32(acc[4 * h]), tc::to_tf32(acc[4 * h + 1]), tc::to_tf32(acc[4 * h + 2]),
+                   tc::to_tf32(acc[4 * h + 3]));
 }
 
 // Warp roles of the persistent tile kernel (32 warps):
-//   warps 0..26  producers: claim kQuad of this CTA's items at a time, build
-//                their T rows on chip, and put each finished row into the next
-//                free slot of the open T buffer, recording its destination;
-//                MMA tiles are thus filled in completion order, so a long
-//                segment delays only its own row, never a whole tile;
-//   warp 27      MMA issuer: waits full[b] (128 rows placed) and free[b]
-//                (buffer's previous accumulator drained), issues the tile's
-//                K/8 tcgen05.mma into TMEM accumulator b, commits to mma[b];
+//   warps 0..26  producers: claim G consecutive items of this CTA's item
+//                tiles at a time (in order), build their T rows with one lane
+//                group per row, and store each row into its item's slot of
+//                the tile's T buffer with its destination; one mbarrier
+//                arrival per claim;
+//   warp 27      MMA issuer: waits full[b] (every claim of the tile placed)
+//                and free[b] (buffer's previous accumulator drained), issues
+//                the tile's K/8 tcgen05.mma into TMEM accumulator b, commits
+//                to mma[b];
 //   warps 28..31 epilogue: wait mma[b], read TMEM lane quadrant (warp % 4),
 //                write A rows or partial rows, arrive free[b].
-// Slot tile n uses buffer n % NBUF; a producer fills it only after the MMAs
-// of tile n - NBUF completed.  Producers may run ahead further than an
-// mbarrier's phase parity can tell apart, so they wait on mma_tiles_done, a
-// monotonic count of completed tiles that the epilogue publishes (release)
-// once all four epilogue warps have read the tile's row destinations.
-// Every wait is bounded; a timeout raises kErrTimeout and the CTA winds down.
+// Item tile n uses buffer n % NBUF; a producer stores into it only after the
+// MMAs of tile n - NBUF completed.  Claims are taken in order, so the claim a
+// producer waits on belongs to an earlier tile, which only needs earlier
+// claims (no cycle).  Producers wait on mma_tiles_done, a monotonic count of
+// completed tiles that the epilogue publishes (release) once all four
+// epilogue warps have read the tile's row destinations.  Every wait is
+// bounded; a timeout raises kErrTimeout and the CTA winds down.
 constexpr int kProducerWarps = 27;
 constexpr int kMmaWarp = 27;  // warps 28..31: epilogue
 
@@ -345,7 +255,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   static_assert(L % 32 == 0 && L >= 32 && L <= 256, "L must be a multiple of 32 in [32, 256]");
   static_assert(kTcThreads == 1024, "32 warps: 27 producers, 1 MMA, 4 epilogue");
   using PL = ProdLayout<K>;
-  constexpr int F = PL::F;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
   constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
@@ -354,7 +263,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ uint64_t full_bar[NBUF], mma_bar[NBUF], free_bar[NBUF];
   __shared__ int2 dest[NBUF][kTcRows];  // per slot: (A row, partial slot); x < 0 = padding
   __shared__ uint32_t tmem_base;
-  __shared__ int claim, fill, fail_flag, mma_tiles_done;
+  __shared__ int claim, fail_flag, mma_tiles_done;
   __shared__ int last_commit[NBUF];     // last tile committed to each accumulator (-1: none)
   uint8_t* sT = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sD = sT + NBUF * TBYTES;
@@ -366,14 +275,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   if (tid == 0) {
     for (int b = 0; b < NBUF; ++b) {
-      tc::mbar_init(&full_bar[b], kTcRows);
+      tc::mbar_init(&full_bar[b], kTcRows / PL::G);  // one arrival per claim
       tc::mbar_init(&mma_bar[b], 1);
       tc::mbar_init(&free_bar[b], 4);
       last_commit[b] = -1;
     }
     tc::fence_mbar_init();
     claim = 0;
-    fill = 0;
     fail_flag = 0;
     mma_tiles_done = 0;
   }
@@ -402,81 +310,59 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int64_t ntiles = (nitems + kTcRows - 1) / kTcRows;
   // this CTA's items: rows of item tiles blockIdx.x + j * gridDim.x, j < nlocal
   const int nlocal = (int)(ntiles > blockIdx.x ? (ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0);
-  int total_rows = nlocal * kTcRows;
-  if (nlocal > 0 && (int64_t)blockIdx.x + (int64_t)(nlocal - 1) * gridDim.x == ntiles - 1)
-    total_rows -= (int)(ntiles * kTcRows - nitems);  // the global last item tile is partial
-  const int pad = nlocal * kTcRows - total_rows;      // padding slots of the last slot tile
 
   if (warp < kProducerWarps) {
     // ---------------- producers ----------------
-    constexpr int QPT = kTcRows / kQuad;  // claims per item tile
-    // claim c covers local item tile c / QPT, rows (c % QPT) * kQuad + 0..kQuad-1;
-    // lane q < kQuad loads the record of row q (x < 0: past the last item)
-    auto load_claim = [&](int c, int4& rec) {
-      rec = make_int4(-1, 0, 0, -1);
-      const int64_t item =
-          ((int64_t)blockIdx.x + (int64_t)(c / QPT) * gridDim.x) * kTcRows + (c % QPT) * kQuad + lane;
-      if (c / QPT < nlocal && lane < kQuad && item < nitems)
-        rec = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
+    // Claim c covers slots (c % CPT) * G + g, g < G, of local item tile
+    // c / CPT; group g of the warp builds the T row of item slot g: it
+    // gathers the row first, then waits for its buffer to be free (the MMAs
+    // of tile c / CPT - NBUF completed and their destinations read), stores
+    // the row and its destination, and lane 0 arrives once for the claim.
+    constexpr int VPL = PL::VPL, G = PL::G, CPT = kTcRows / G;
+    const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
+    const int nclaims = nlocal * CPT;
+    auto claim_item = [&](int c) -> int64_t {
+      return ((int64_t)blockIdx.x + (int64_t)(c / CPT) * gridDim.x) * kTcRows + (c % CPT) * G + g;
     };
-    // hands a finished T row of claimed item q to the next free slot
-    int4 rec = make_int4(-1, 0, 0, -1);
-    auto emit = [&](int q, const Frag<F>& acc) -> bool {
-      const int rx = __shfl_sync(0xffffffffu, rec.x, q), rw = __shfl_sync(0xffffffffu, rec.w, q);
-      if (rx < 0) return true;  // past the last item: no row
-      int slot = 0;
-      if (lane == 0) slot = atomicAdd(&fill, 1);
-      slot = __shfl_sync(0xffffffffu, slot, 0);
-      const int n = slot / kTcRows, s = slot % kTcRows, b = n % NBUF;
-      if (n >= NBUF) {  // buffer b is free once the MMAs of slot tile n - NBUF completed
-        const bool ok = count_wait_timeout(&mma_tiles_done, n - NBUF + 1);
-        if (!__all_sync(0xffffffffu, ok)) return false;
+    auto load_rec = [&](int c) -> int4 {
+      int4 r = make_int4(-1, 0, 0, -1);
+      if (c < nclaims) {
+        const int64_t item = claim_item(c);
+        if (item < nitems) r = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
       }
-      store_t_row<K>(sT + b * TBYTES, s, lane, acc);
-      if (lane == 0) dest[b][s] = make_int2(rx, rw);
-      tc::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        if (slot == total_rows - 1 && pad > 0) {  // the last row: pad the final slot tile
-          for (int i = s + 1; i < kTcRows; ++i) dest[b][i] = make_int2(-1, -1);
-          tc::mbar_arrive_n(&full_bar[b], 1 + pad);
-        } else {
-          tc::mbar_arrive(&full_bar[b]);
-        }
-      }
-      return true;
+      return r;
     };
     int x = 0;
     if (lane == 0) x = atomicAdd(&claim, 1);
     int cl = __shfl_sync(0xffffffffu, x, 0);
-    load_claim(cl, rec);
-    while (cl / QPT < nlocal) {
+    int4 rec = load_rec(cl);
+    while (cl < nclaims) {
       x = 0;
       if (lane == 0) x = atomicAdd(&claim, 1);
       const int cl_next = __shfl_sync(0xffffffffu, x, 0);
-      int4 rec_next;
-      load_claim(cl_next, rec_next);  // loads while this claim is built
-      bool ok = true;
-      if (MODE == kSegments) {
-        // items past the last one get an empty range at the end of the last valid item
-        const unsigned valid = __ballot_sync(0xffffffffu, lane < kQuad && rec.x >= 0) & ((1u << kQuad) - 1u);
-        const int nvalid = __popc(valid);
-        const int start0 = __shfl_sync(0xffffffffu, rec.y, 0);
-        const int last_end = __shfl_sync(0xffffffffu, rec.z, nvalid > 0 ? nvalid - 1 : 0);
-        const int my_end = rec.x >= 0 ? rec.z : (nvalid > 0 ? last_end : start0);
-        ok = build_quad<K, PL::U>(my_end, nvalid > 0 ? start0 : 0, lane, crd, vals, X, emit);
-      } else {
-#pragma unroll
-        for (int q = 0; q < kQuad && ok; ++q) {
-          const int rx = __shfl_sync(0xffffffffu, rec.x, q);
-          const Frag<F> acc = rx >= 0 ? ldg_frag<F>(X + (int64_t)rx * K + F * lane) : zero_frag<F>();
-          ok = emit(q, acc);
+      const int4 rec_next = load_rec(cl_next);  // loads while this claim is built
+      float acc[VPL];
+      zero_vec(acc);
+      if (rec.x >= 0) {
+        if (MODE == kSegments)
+          gather_acc<VPL, PL::U>(acc, crd, vals, rec.y, rec.z, X, K, col);
+        else
+          ldg_vec<VPL>(acc, X + (int64_t)rec.x * K + col);
+      }
+      __syncwarp();
+      const int j = cl / CPT, b = j % NBUF, s = (cl % CPT) * G + g;
+      if (j >= NBUF) {
+        const bool ok = count_wait_timeout(&mma_tiles_done, j - NBUF + 1);
+        if (!__all_sync(0xffffffffu, ok)) {
+          atomicOr(&fail_flag, 1);
+          break;
         }
       }
-      if (!ok) {
-        atomicOr(&fail_flag, 1);
-        break;
-      }
+      store_t_part<VPL>(sT + b * TBYTES, s, col, acc);
+      if (lane % PL::GS == 0) dest[b][s] = make_int2(rec.x, rec.w);
+      tc::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&full_bar[b]);
       cl = cl_next;
       rec = rec_next;
     }
