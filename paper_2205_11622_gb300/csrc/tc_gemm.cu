@@ -196,6 +196,9 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 #ifndef SLNR_TC_UNROLL
 #define SLNR_TC_UNROLL 8  // gathered rows in flight per lane group
 #endif
+#ifndef SLNR_TC_DENSE_ROWS
+#define SLNR_TC_DENSE_ROWS 4  // DENSE mode: rows of T loaded at once per lane group
+#endif
 
 // Producer layout: a T row is built by a group of GS = K / VPL lanes, lane gl
 // of the group holding the VPL columns [VPL*gl, VPL*gl + VPL), loaded as
@@ -275,7 +278,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   if (tid == 0) {
     for (int b = 0; b < NBUF; ++b) {
-      tc::mbar_init(&full_bar[b], kTcRows / PL::G);  // one arrival per claim
+      tc::mbar_init(&full_bar[b], kTcRows / (PL::G * (MODE == kSegments ? 1 : SLNR_TC_DENSE_ROWS)));  // one arrival per claim
       tc::mbar_init(&mma_bar[b], 1);
       tc::mbar_init(&free_bar[b], 4);
       last_commit[b] = -1;
@@ -313,44 +316,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (warp < kProducerWarps) {
     // ---------------- producers ----------------
-    // Claim c covers slots (c % CPT) * G + g, g < G, of local item tile
-    // c / CPT; group g of the warp builds the T row of item slot g: it
-    // gathers the row first, then waits for its buffer to be free (the MMAs
-    // of tile c / CPT - NBUF completed and their destinations read), stores
-    // the row and its destination, and lane 0 arrives once for the claim.
-    constexpr int VPL = PL::VPL, G = PL::G, CPT = kTcRows / G;
+    // A claim covers IPC = G * R consecutive items of local item tile c / CPT:
+    // lane group g builds the T rows of items g, g + G, ..., g + (R-1) G of
+    // the claim (R = 1 gathered segment, or R = U rows of a materialised T in
+    // DENSE mode, all loads in flight at once).  It builds the rows first,
+    // then waits for its buffer to be free (the MMAs of tile c / CPT - NBUF
+    // completed and their destinations read), stores the rows and their
+    // destinations, and lane 0 arrives once for the claim.
+    constexpr int VPL = PL::VPL, G = PL::G, R = MODE == kSegments ? 1 : SLNR_TC_DENSE_ROWS;
+    constexpr int IPC = G * R, CPT = kTcRows / IPC;
+    static_assert(kTcRows % IPC == 0, "claims tile the item tile");
     const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
     const int nclaims = nlocal * CPT;
-    auto claim_item = [&](int c) -> int64_t {
-      return ((int64_t)blockIdx.x + (int64_t)(c / CPT) * gridDim.x) * kTcRows + (c % CPT) * G + g;
-    };
-    auto load_rec = [&](int c) -> int4 {
-      int4 r = make_int4(-1, 0, 0, -1);
+    auto load_rec = [&](int c, int r) -> int4 {
+      int4 rv = make_int4(-1, 0, 0, -1);
       if (c < nclaims) {
-        const int64_t item = claim_item(c);
-        if (item < nitems) r = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
+        const int64_t item =
+            ((int64_t)blockIdx.x + (int64_t)(c / CPT) * gridDim.x) * kTcRows + (c % CPT) * IPC + r * G + g;
+        if (item < nitems) rv = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
       }
-      return r;
+      return rv;
     };
     int x = 0;
     if (lane == 0) x = atomicAdd(&claim, 1);
     int cl = __shfl_sync(0xffffffffu, x, 0);
-    int4 rec = load_rec(cl);
+    int4 rec = load_rec(cl, 0);  // segment record (R = 1)
     while (cl < nclaims) {
       x = 0;
       if (lane == 0) x = atomicAdd(&claim, 1);
       const int cl_next = __shfl_sync(0xffffffffu, x, 0);
-      const int4 rec_next = load_rec(cl_next);  // loads while this claim is built
-      float acc[VPL];
-      zero_vec(acc);
-      if (rec.x >= 0) {
-        if (MODE == kSegments)
-          gather_acc<VPL, PL::U>(acc, crd, vals, rec.y, rec.z, X, K, col);
-        else
-          ldg_vec<VPL>(acc, X + (int64_t)rec.x * K + col);
+      float acc[R][VPL];
+      int2 dst0 = make_int2(-1, -1);  // destination of the segment (R = 1)
+      if constexpr (MODE == kSegments) {
+        const int4 rec_next = load_rec(cl_next, 0);  // loads while this claim is built
+        zero_vec(acc[0]);
+        if (rec.x >= 0) gather_acc<VPL, PL::U>(acc[0], crd, vals, rec.y, rec.z, X, K, col);
+        dst0 = make_int2(rec.x, rec.w);
+        rec = rec_next;
+      } else {
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          const int4 rr = load_rec(cl, r);
+          if (rr.x >= 0) ldg_vec<VPL>(acc[r], X + (int64_t)rr.x * K + col); else zero_vec(acc[r]);
+        }
       }
       __syncwarp();
-      const int j = cl / CPT, b = j % NBUF, s = (cl % CPT) * G + g;
+      const int j = cl / CPT, b = j % NBUF, s0 = (cl % CPT) * IPC + g;
       if (j >= NBUF) {
         const bool ok = count_wait_timeout(&mma_tiles_done, j - NBUF + 1);
         if (!__all_sync(0xffffffffu, ok)) {
@@ -358,13 +369,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           break;
         }
       }
-      store_t_part<VPL>(sT + b * TBYTES, s, col, acc);
-      if (lane % PL::GS == 0) dest[b][s] = make_int2(rec.x, rec.w);
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        store_t_part<VPL>(sT + b * TBYTES, s0 + r * G, col, acc[r]);
+        if (lane % PL::GS == 0)
+          dest[b][s0 + r * G] = MODE == kSegments ? dst0 : make_int2(load_rec(cl, r).x, -1);
+      }
       tc::fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&full_bar[b]);
       cl = cl_next;
-      rec = rec_next;
     }
   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
