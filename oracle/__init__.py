@@ -1,7 +1,7 @@
 """ORACLE -- test infrastructure, not part of the library.
 
 ctypes binding of ``oracle.c``: the plain, single-threaded fp64 CPU evaluation
-of the four composite sparse expressions (SparseLNR, Sec. 6.2), in the loop
+of the composite sparse expressions of SparseLNR's benchmarks (Sec. 6.2), in the loop
 order that the paper's fusion-after-distribution transformation produces
 (Sec. 4.2, Algorithm 1).  Only ``tests/``, ``__graft_entry__.smoke()`` and the
 CPU-baseline leg of ``bench.py`` may import this package.  It never imports or
@@ -74,6 +74,12 @@ class Oracle:
         lib.oracle_spttm_ttm.restype = ctypes.c_int
         lib.oracle_spttm_ttm_pattern.argtypes = [i32, P, P, P, P, P, P, P]
         lib.oracle_spttm_ttm_pattern.restype = ctypes.c_int64
+        lib.oracle_sddmm_spmm_gemm.argtypes = [i32, i32, P, P, P, P, P, i32, P, i32, P, i32, i64, P, P, P]
+        lib.oracle_sddmm_spmm_gemm.restype = ctypes.c_int
+        lib.oracle_mttkrp_gemm.argtypes = [i32, i32, i32, i32, P, P, P, P, P, P, P, P, i32, P, i32, i64, P, P, P]
+        lib.oracle_mttkrp_gemm.restype = ctypes.c_int
+        lib.oracle_spmmh_gemm.argtypes = [i32, i32, P, P, P, P, P, i32, P, i32, i64, P, P, P]
+        lib.oracle_spmmh_gemm.restype = ctypes.c_int
         self.lib = lib
 
     @staticmethod
@@ -148,6 +154,48 @@ class Oracle:
             raise ValueError("oracle_spttm_ttm_pattern: malformed input")
         return p1, c1[:ns], p2, c2[:got]
 
+    def sddmm_spmm_gemm(self, nrows, ncols, pos, crd, vals, C, D, F, W, rows=None):
+        """A(i,m) = sum_{j,k,l} B(i,j) C(i,k) D(j,k) F(j,l) W(l,m) for the selected rows i."""
+        pos, crd, vals = _i32(pos), _i32(crd), _f32(vals)
+        C, D, F, W = _f32(C), _f32(D), _f32(F), _f32(W)
+        K, L, M = C.shape[1], F.shape[1], W.shape[1]
+        assert C.shape[0] == nrows and D.shape == (ncols, K) and F.shape[0] == ncols and W.shape[0] == L
+        sel, n = self._sel(rows, nrows)
+        A = np.empty((n, M)); Aa = np.empty((n, M))
+        rc = self.lib.oracle_sddmm_spmm_gemm(nrows, ncols, _p(pos), _p(crd), _p(vals), _p(C), _p(D), K, _p(F), L,
+                                             _p(W), M, n, _p(sel), _p(A), _p(Aa))
+        if rc != 0:
+            raise ValueError("oracle_sddmm_spmm_gemm: malformed input")
+        return A, Aa
+
+    def mttkrp_gemm(self, dims, crd1, pos2, crd2, pos3, crd3, vals, C, D, E, rows=None):
+        """A(i,m) = sum_{j,k,l} B(i,j,k) C(j,l) D(k,l) E(l,m) for the selected rows i."""
+        crd1, pos2, crd2, pos3, crd3 = map(_i32, (crd1, pos2, crd2, pos3, crd3))
+        vals, C, D, E = _f32(vals), _f32(C), _f32(D), _f32(E)
+        L, M = C.shape[1], E.shape[1]
+        assert C.shape[0] == dims[1] and D.shape == (dims[2], L) and E.shape[0] == L
+        sel, n = self._sel(rows, dims[0])
+        A = np.empty((n, M)); Aa = np.empty((n, M))
+        rc = self.lib.oracle_mttkrp_gemm(dims[0], dims[1], dims[2], crd1.shape[0], _p(crd1), _p(pos2), _p(crd2),
+                                         _p(pos3), _p(crd3), _p(vals), _p(C), _p(D), L, _p(E), M, n, _p(sel),
+                                         _p(A), _p(Aa))
+        if rc != 0:
+            raise ValueError("oracle_mttkrp_gemm: malformed input")
+        return A, Aa
+
+    def spmmh_gemm(self, nrows, ncols, pos, crd, vals, C, D, E, rows=None):
+        """A(i,l) = sum_{k,j} B(i,k) C(k,j) D(k,j) E(j,l) for the selected rows i."""
+        pos, crd, vals, C, D, E = _i32(pos), _i32(crd), _f32(vals), _f32(C), _f32(D), _f32(E)
+        J, L = C.shape[1], E.shape[1]
+        assert C.shape[0] == ncols and D.shape == C.shape and E.shape[0] == J
+        sel, n = self._sel(rows, nrows)
+        A = np.empty((n, L)); Aa = np.empty((n, L))
+        rc = self.lib.oracle_spmmh_gemm(nrows, ncols, _p(pos), _p(crd), _p(vals), _p(C), _p(D), J, _p(E), L, n,
+                                        _p(sel), _p(A), _p(Aa))
+        if rc != 0:
+            raise ValueError("oracle_spmmh_gemm: malformed input")
+        return A, Aa
+
     # --- convenience on workloads.Workload objects ---------------------------------
     def run(self, w, rows=None):
         B, d = w.B, w.dense
@@ -159,6 +207,14 @@ class Oracle:
             return self.mttkrp(B.dims, B.crd1, B.pos2, B.crd2, B.pos3, B.crd3, B.vals, d["C"], d["D"], rows)
         if w.op == "spttm_ttm":
             return self.spttm_ttm(B.dims[2], B.pos3, B.crd3, B.vals, d["C"], d["D"], rows)
+        if w.op == "sddmm_spmm_gemm":
+            return self.sddmm_spmm_gemm(B.nrows, B.ncols, B.pos, B.crd, B.vals, d["C"], d["D"], d["F"], d["W"],
+                                        rows)
+        if w.op == "mttkrp_gemm":
+            return self.mttkrp_gemm(B.dims, B.crd1, B.pos2, B.crd2, B.pos3, B.crd3, B.vals, d["C"], d["D"], d["E"],
+                                    rows)
+        if w.op == "spmmh_gemm":
+            return self.spmmh_gemm(B.nrows, B.ncols, B.pos, B.crd, B.vals, d["C"], d["D"], d["E"], rows)
         raise ValueError(w.op)
 
 

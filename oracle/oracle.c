@@ -323,3 +323,242 @@ int64_t oracle_spttm_ttm_pattern(int32_t nslices, const int32_t *crd1, const int
   A_pos1[1] = nslices;
   return nf;
 }
+
+/*
+ * <SDDMM,SpMM,GEMM> (Sec. 6.2): A(i,m) = sum_{j,k,l} B(i,j) C(i,k) D(j,k) F(j,l) W(l,m)
+ * -- the sampled products B(i,j) <C(i,:), D(j,:)>, a neighbour sum of F's rows
+ * with those weights, and the product with W.
+ *
+ * Algorithm 1 applied recursively (Sec. 4.2 notes it can be reapplied to the
+ * producer): removing W leaves producer P(i,l) = sum_j B(i,j) <C(i,:),D(j,:)>
+ * F(j,l) (loops i, j, k, l) and consumer A(i,m) = sum_l P(i,l) W(l,m) (loops
+ * i, l, m): common prefix {i}, temporary a vector over l per row.  The
+ * producer is itself <SDDMM,SpMM>, whose temporary is a scalar per stored
+ * (i,j).  So, per row i: for each stored j, y = B(i,j) <C(i,:), D(j,:)>,
+ * t(l) += y F(j,l); then A(i,m) = sum_l t(l) W(l,m).
+ *
+ * B: nrows x ncols CSR.  C: nrows x K.  D: ncols x K.  F: ncols x L.
+ * W: L x M.  Output rows as for oracle_spmm_gemm; A / A_abs are nsel x M.
+ */
+int oracle_sddmm_spmm_gemm(int32_t nrows, int32_t ncols, const int32_t *pos, const int32_t *crd,
+                           const float *vals, const float *C, const float *D, int32_t K, const float *F,
+                           int32_t L, const float *W, int32_t M, int64_t nsel, const int32_t *rows,
+                           double *A, double *A_abs) {
+  double *t = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  double *ta = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  if (!t || !ta) {
+    free(t);
+    free(ta);
+    return -1;
+  }
+  int rc = 0;
+  for (int64_t s = 0; s < nsel && rc == 0; ++s) {
+    const int32_t i = rows ? rows[s] : (int32_t)s;
+    if (!csr_row_ok(nrows, pos, i)) {
+      rc = -1;
+      break;
+    }
+    for (int32_t l = 0; l < L; ++l) {
+      t[l] = 0.0;
+      ta[l] = 0.0;
+    }
+    for (int32_t p = pos[i]; p < pos[i + 1]; ++p) {
+      const int32_t j = crd[p];
+      if (j < 0 || j >= ncols) {
+        rc = -1;
+        break;
+      }
+      const double b = (double)vals[p];
+      /* innermost producer: the scalar y = B(i,j) sum_k C(i,k) D(j,k) */
+      double y = 0.0, ya = 0.0;
+      for (int32_t k = 0; k < K; ++k) {
+        const double c = (double)C[(int64_t)i * K + k];
+        const double d = (double)D[(int64_t)j * K + k];
+        y += b * c * d;
+        ya += fabs(b) * fabs(c) * fabs(d);
+      }
+      /* its consumer, the outer producer: t(l) += y F(j,l) */
+      for (int32_t l = 0; l < L; ++l) {
+        const double f = (double)F[(int64_t)j * L + l];
+        t[l] += y * f;
+        ta[l] += ya * fabs(f);
+      }
+    }
+    /* outer consumer: A(i,m) = sum_l t(l) W(l,m) */
+    for (int32_t m = 0; m < M; ++m) {
+      double acc = 0.0, acc_abs = 0.0;
+      for (int32_t l = 0; l < L; ++l) {
+        const double w = (double)W[(int64_t)l * M + m];
+        acc += t[l] * w;
+        acc_abs += ta[l] * fabs(w);
+      }
+      A[s * M + m] = acc;
+      A_abs[s * M + m] = acc_abs;
+    }
+  }
+  free(t);
+  free(ta);
+  return rc;
+}
+
+/*
+ * <MTTKRP,GEMM> (Sec. 6.2), with the index names of the C interface:
+ * A(i,m) = sum_{j,k,l} B(i,j,k) C(j,l) D(k,l) E(l,m) -- MTTKRP followed by a
+ * product with E (the paper prints A_im = sum B_ikl C_lj D_kj E_jm; its rank
+ * index j is l here, as in oracle_mttkrp).
+ *
+ * Algorithm 1, applied twice: removing E leaves producer P(i,l) = MTTKRP and
+ * consumer A(i,m) = sum_l P(i,l) E(l,m), common prefix {i}, temporary u(l)
+ * per slice; the producer splits again as in oracle_mttkrp into t(l) per
+ * fiber.  Per slice i: u(l) = sum_j t_j(l) C(j,l) with t_j(l) = sum_k
+ * B(i,j,k) D(k,l); then A(i,m) = sum_l u(l) E(l,m).
+ *
+ * B: CSF (as oracle_mttkrp), dims d0 x d1 x d2.  C: d1 x L.  D: d2 x L.
+ * E: L x M.  A / A_abs: nsel x M for output rows rows[0..nsel) (or
+ * 0..nsel-1); a row with no slice is zero.
+ */
+int oracle_mttkrp_gemm(int32_t d0, int32_t d1, int32_t d2, int32_t nslices, const int32_t *crd1,
+                       const int32_t *pos2, const int32_t *crd2, const int32_t *pos3,
+                       const int32_t *crd3, const float *vals, const float *C, const float *D,
+                       int32_t L, const float *E, int32_t M, int64_t nsel, const int32_t *rows,
+                       double *A, double *A_abs) {
+  double *t = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  double *ta = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  double *u = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  double *ua = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  if (!t || !ta || !u || !ua) {
+    free(t);
+    free(ta);
+    free(u);
+    free(ua);
+    return -1;
+  }
+  int rc = 0;
+  for (int64_t s = 0; s < nsel && rc == 0; ++s) {
+    const int32_t i = rows ? rows[s] : (int32_t)s;
+    if (i < 0 || i >= d0) {
+      rc = -1;
+      break;
+    }
+    for (int32_t l = 0; l < L; ++l) {
+      u[l] = 0.0;
+      ua[l] = 0.0;
+    }
+    for (int32_t q = 0; q < nslices && rc == 0; ++q) {
+      if (crd1[q] != i) continue;
+      for (int32_t f = pos2[q]; f < pos2[q + 1] && rc == 0; ++f) {
+        const int32_t j = crd2[f];
+        if (j < 0 || j >= d1) {
+          rc = -1;
+          break;
+        }
+        /* fiber producer: t(l) = sum_k B(i,j,k) D(k,l) */
+        for (int32_t l = 0; l < L; ++l) {
+          t[l] = 0.0;
+          ta[l] = 0.0;
+        }
+        for (int32_t p = pos3[f]; p < pos3[f + 1]; ++p) {
+          const int32_t k = crd3[p];
+          if (k < 0 || k >= d2) {
+            rc = -1;
+            break;
+          }
+          const double b = (double)vals[p];
+          for (int32_t l = 0; l < L; ++l) {
+            const double d = (double)D[(int64_t)k * L + l];
+            t[l] += b * d;
+            ta[l] += fabs(b) * fabs(d);
+          }
+        }
+        /* fiber consumer, slice producer: u(l) += t(l) C(j,l) */
+        for (int32_t l = 0; l < L; ++l) {
+          const double c = (double)C[(int64_t)j * L + l];
+          u[l] += t[l] * c;
+          ua[l] += ta[l] * fabs(c);
+        }
+      }
+    }
+    /* slice consumer: A(i,m) = sum_l u(l) E(l,m) */
+    for (int32_t m = 0; m < M; ++m) {
+      double acc = 0.0, acc_abs = 0.0;
+      for (int32_t l = 0; l < L; ++l) {
+        const double e = (double)E[(int64_t)l * M + m];
+        acc += u[l] * e;
+        acc_abs += ua[l] * fabs(e);
+      }
+      A[s * M + m] = acc;
+      A_abs[s * M + m] = acc_abs;
+    }
+  }
+  free(t);
+  free(ta);
+  free(u);
+  free(ua);
+  return rc;
+}
+
+/*
+ * <SpMMH,GEMM> (Sec. 6.2): A(i,l) = sum_{k,j} B(i,k) C(k,j) D(k,j) E(j,l) -- a
+ * sparse matrix times the Hadamard product of two dense matrices, then a
+ * product with E.
+ *
+ * Algorithm 1 removes E: producer T'(i,j) = sum_k B(i,k) C(k,j) D(k,j) (loops
+ * i, k, j), consumer A(i,l) = sum_j T'(i,j) E(j,l) (loops i, j, l).  Common
+ * prefix {i}; below it j is shared, so the temporary is a vector over j per
+ * row, as in <SpMM,GEMM>.
+ *
+ * B: nrows x ncols CSR (row i, column k).  C, D: ncols x J.  E: J x L.
+ * Output rows as for oracle_spmm_gemm; A / A_abs are nsel x L.
+ */
+int oracle_spmmh_gemm(int32_t nrows, int32_t ncols, const int32_t *pos, const int32_t *crd,
+                      const float *vals, const float *C, const float *D, int32_t J, const float *E,
+                      int32_t L, int64_t nsel, const int32_t *rows, double *A, double *A_abs) {
+  double *t = (double *)malloc(sizeof(double) * (size_t)(J > 0 ? J : 1));
+  double *ta = (double *)malloc(sizeof(double) * (size_t)(J > 0 ? J : 1));
+  if (!t || !ta) {
+    free(t);
+    free(ta);
+    return -1;
+  }
+  int rc = 0;
+  for (int64_t s = 0; s < nsel && rc == 0; ++s) {
+    const int32_t i = rows ? rows[s] : (int32_t)s;
+    if (!csr_row_ok(nrows, pos, i)) {
+      rc = -1;
+      break;
+    }
+    /* producer: t(j) = sum_k B(i,k) C(k,j) D(k,j) */
+    for (int32_t j = 0; j < J; ++j) {
+      t[j] = 0.0;
+      ta[j] = 0.0;
+    }
+    for (int32_t p = pos[i]; p < pos[i + 1]; ++p) {
+      const int32_t k = crd[p];
+      if (k < 0 || k >= ncols) {
+        rc = -1;
+        break;
+      }
+      const double b = (double)vals[p];
+      for (int32_t j = 0; j < J; ++j) {
+        const double c = (double)C[(int64_t)k * J + j];
+        const double d = (double)D[(int64_t)k * J + j];
+        t[j] += b * c * d;
+        ta[j] += fabs(b) * fabs(c) * fabs(d);
+      }
+    }
+    /* consumer: A(i,l) = sum_j t(j) E(j,l) */
+    for (int32_t l = 0; l < L; ++l) {
+      double acc = 0.0, acc_abs = 0.0;
+      for (int32_t j = 0; j < J; ++j) {
+        const double e = (double)E[(int64_t)j * L + l];
+        acc += t[j] * e;
+        acc_abs += ta[j] * fabs(e);
+      }
+      A[s * L + l] = acc;
+      A_abs[s * L + l] = acc_abs;
+    }
+  }
+  free(t);
+  free(ta);
+  return rc;
+}

@@ -373,11 +373,202 @@ def check_spttm_ttm(orc, seed=4, square_lm=False):
     return fails
 
 
+# --------------------------------------------------------------------------
+# <SDDMM,SpMM,GEMM>: A(i,m) = sum_{j,k,l} B(i,j) C(i,k) D(j,k) F(j,l) W(l,m)
+
+def check_sddmm_spmm_gemm(orc, seed=5):
+    fails = []
+    rng = np.random.default_rng(seed)
+    nrows, ncols, K, L, M = 7, 8, 3, 4, 5
+    pos, crd, vals = rand_csr(rng, nrows, ncols, 0.4, empty_rows=(4,))
+    C, D = f32(rng, (nrows, K)), f32(rng, (ncols, K))
+    F, W = f32(rng, (ncols, L)), f32(rng, (L, M))
+    Bd = csr_dense(nrows, ncols, pos, crd, vals)
+    C64, D64, F64, W64 = (x.astype(np.float64) for x in (C, D, F, W))
+    A, Aa = orc.sddmm_spmm_gemm(nrows, ncols, pos, crd, vals, C, D, F, W)
+    ref = np.einsum("ij,ik,jk,jl,lm->im", Bd, C64, D64, F64, W64)
+    ref_abs = np.einsum("ij,ik,jk,jl,lm->im", *(np.abs(x) for x in (Bd, C64, D64, F64, W64)))
+    if not _close(A, ref, ref_abs):
+        fails.append("sddmm_spmm_gemm brute force")
+    if not _close(Aa, ref_abs, ref_abs):
+        fails.append("sddmm_spmm_gemm magnitude companion")
+    if not np.all(A[4] == 0):
+        fails.append("sddmm_spmm_gemm empty row")
+    # the paper's reading of the chain (Sec. 6.2): attention values on the
+    # edges, the features times the weights, then the neighbour sum
+    Y = Bd * (C64 @ D64.T)
+    if not _close(A, Y @ (F64 @ W64), ref_abs):
+        fails.append("sddmm_spmm_gemm equals SDDMM, then SpMM with F.W")
+    # W = I: <SDDMM,SpMM>, here by scipy's sparse product of the sampled matrix
+    Ai, Aia = orc.sddmm_spmm_gemm(nrows, ncols, pos, crd, vals, C, D, F, np.eye(L, dtype=np.float32))
+    Ys = sp.csr_matrix((vals.astype(np.float64) * np.einsum("pk,pk->p", C64[np.repeat(np.arange(nrows), np.diff(pos))],
+                                                             D64[crd]), crd, pos), shape=(nrows, ncols))
+    if not _close(Ai, Ys @ F64, Aia):
+        fails.append("sddmm_spmm_gemm W=I is SDDMM-SpMM")
+    # exact integers
+    pos_i, crd_i, vals_i = rand_csr(rng, 3, 4, 0.6, values="int")
+    Ci, Di, Fi, Wi = ints(rng, (3, 2)), ints(rng, (4, 2)), ints(rng, (4, 3)), ints(rng, (3, 2))
+    Bi = csr_dense(3, 4, pos_i, crd_i, vals_i).astype(int).tolist()
+    Cl, Dl, Fl, Wl = (x.astype(int).tolist() for x in (Ci, Di, Fi, Wi))
+    exact = [[sum(Bi[i][j] * Cl[i][k] * Dl[j][k] * Fl[j][l] * Wl[l][m]
+                  for j in range(4) for k in range(2) for l in range(3)) for m in range(2)] for i in range(3)]
+    Ae, _ = orc.sddmm_spmm_gemm(3, 4, pos_i, crd_i, vals_i, Ci, Di, Fi, Wi)
+    if not np.array_equal(Ae, np.array(exact, dtype=np.float64)):
+        fails.append("sddmm_spmm_gemm exact integers")
+    # linearity in C, F and W
+    Cy, C2 = dyadic(rng, (nrows, K)), dyadic(rng, (nrows, K))
+    Fy, F2 = dyadic(rng, (ncols, L)), dyadic(rng, (ncols, L))
+    Wy, W2 = dyadic(rng, (L, M)), dyadic(rng, (L, M))
+    a, b = 0.5, -1.75
+    run = lambda c, f, w: orc.sddmm_spmm_gemm(nrows, ncols, pos, crd, vals, c, D, f, w)
+    A0, s0 = run(Cy, Fy, Wy)
+    for name, args2, argsab in (("C", (C2, Fy, Wy), (combo(a, Cy, b, C2), Fy, Wy)),
+                                ("F", (Cy, F2, Wy), (Cy, combo(a, Fy, b, F2), Wy)),
+                                ("W", (Cy, Fy, W2), (Cy, Fy, combo(a, Wy, b, W2)))):
+        Aab, sab = run(*argsab)
+        A2, _ = run(*args2)
+        if not _close(Aab, a * A0 + b * A2, sab + s0):
+            fails.append(f"sddmm_spmm_gemm linear in {name}")
+    rows = np.array([6, 4, 0], np.int32)
+    As, _ = orc.sddmm_spmm_gemm(nrows, ncols, pos, crd, vals, C, D, F, W, rows=rows)
+    if not np.array_equal(As, A[rows]):
+        fails.append("sddmm_spmm_gemm row selection")
+    return fails
+
+
+# --------------------------------------------------------------------------
+# <MTTKRP,GEMM>: A(i,m) = sum_{j,k,l} B(i,j,k) C(j,l) D(k,l) E(l,m)
+
+def check_mttkrp_gemm(orc, seed=6):
+    fails = []
+    rng = np.random.default_rng(seed)
+    dims, L, M = (6, 5, 7), 4, 3
+    csf = rand_csf(rng, dims, 0.25, empty_slice_rows=(2,))
+    C, D, E = f32(rng, (dims[1], L)), f32(rng, (dims[2], L)), f32(rng, (L, M))
+    Bd = csf_dense(dims, *csf)
+    C64, D64, E64 = (x.astype(np.float64) for x in (C, D, E))
+    A, Aa = orc.mttkrp_gemm(dims, *csf, C, D, E)
+    ref = np.einsum("ijk,jl,kl,lm->im", Bd, C64, D64, E64)
+    ref_abs = np.einsum("ijk,jl,kl,lm->im", *(np.abs(x) for x in (Bd, C64, D64, E64)))
+    if not _close(A, ref, ref_abs):
+        fails.append("mttkrp_gemm brute force")
+    if not _close(Aa, ref_abs, ref_abs):
+        fails.append("mttkrp_gemm magnitude companion")
+    if not np.all(A[2] == 0):
+        fails.append("mttkrp_gemm empty slice")
+    # matricised form B_(1) (C kr D) E
+    B1 = Bd.reshape(dims[0], dims[1] * dims[2])
+    KR = (C64[:, None, :] * D64[None, :, :]).reshape(dims[1] * dims[2], L)
+    if not _close(A, B1 @ KR @ E64, ref_abs):
+        fails.append("mttkrp_gemm Khatri-Rao form")
+    # L = 1, C = D = 1: A(i,m) = (sum of slice i) * E(0,m)
+    e1 = f32(rng, (1, M))
+    A1, A1a = orc.mttkrp_gemm(dims, *csf, np.ones((dims[1], 1), np.float32), np.ones((dims[2], 1), np.float32), e1)
+    if not _close(A1, np.outer(Bd.sum(axis=(1, 2)), e1[0].astype(np.float64)), A1a):
+        fails.append("mttkrp_gemm slice sums")
+    # exact integers
+    dims_i = (3, 3, 4)
+    csf_i = rand_csf(rng, dims_i, 0.4, values="int")
+    Ci, Di, Ei = ints(rng, (3, 2)), ints(rng, (4, 2)), ints(rng, (2, 3))
+    Bi = csf_dense(dims_i, *csf_i).astype(int).tolist()
+    Cl, Dl, El = (x.astype(int).tolist() for x in (Ci, Di, Ei))
+    exact = [[sum(Bi[i][j][k] * Cl[j][l] * Dl[k][l] * El[l][m] for j in range(3) for k in range(4) for l in range(2))
+              for m in range(3)] for i in range(3)]
+    Ae, _ = orc.mttkrp_gemm(dims_i, *csf_i, Ci, Di, Ei)
+    if not np.array_equal(Ae, np.array(exact, dtype=np.float64)):
+        fails.append("mttkrp_gemm exact integers")
+    # linearity in C, D and E
+    Cy, C2 = dyadic(rng, (dims[1], L)), dyadic(rng, (dims[1], L))
+    Dy, D2 = dyadic(rng, (dims[2], L)), dyadic(rng, (dims[2], L))
+    Ey, E2 = dyadic(rng, (L, M)), dyadic(rng, (L, M))
+    a, b = -0.5, 2.0
+    run = lambda c, d, e: orc.mttkrp_gemm(dims, *csf, c, d, e)
+    A0, s0 = run(Cy, Dy, Ey)
+    for name, args2, argsab in (("C", (C2, Dy, Ey), (combo(a, Cy, b, C2), Dy, Ey)),
+                                ("D", (Cy, D2, Ey), (Cy, combo(a, Dy, b, D2), Ey)),
+                                ("E", (Cy, Dy, E2), (Cy, Dy, combo(a, Ey, b, E2)))):
+        Aab, sab = run(*argsab)
+        A2, _ = run(*args2)
+        if not _close(Aab, a * A0 + b * A2, sab + s0):
+            fails.append(f"mttkrp_gemm linear in {name}")
+    rows = np.array([5, 2, 0], np.int32)
+    As, _ = orc.mttkrp_gemm(dims, *csf, C, D, E, rows=rows)
+    if not np.array_equal(As, A[rows]):
+        fails.append("mttkrp_gemm row selection")
+    return fails
+
+
+# --------------------------------------------------------------------------
+# <SpMMH,GEMM>: A(i,l) = sum_{k,j} B(i,k) C(k,j) D(k,j) E(j,l)
+
+def check_spmmh_gemm(orc, seed=7):
+    fails = []
+    rng = np.random.default_rng(seed)
+    nrows, ncols, J, L = 6, 9, 4, 5
+    pos, crd, vals = rand_csr(rng, nrows, ncols, 0.4, empty_rows=(1,))
+    C, D, E = f32(rng, (ncols, J)), f32(rng, (ncols, J)), f32(rng, (J, L))
+    Bd = csr_dense(nrows, ncols, pos, crd, vals)
+    C64, D64, E64 = (x.astype(np.float64) for x in (C, D, E))
+    A, Aa = orc.spmmh_gemm(nrows, ncols, pos, crd, vals, C, D, E)
+    ref = np.einsum("ik,kj,kj,jl->il", Bd, C64, D64, E64)
+    ref_abs = np.einsum("ik,kj,kj,jl->il", *(np.abs(x) for x in (Bd, C64, D64, E64)))
+    if not _close(A, ref, ref_abs):
+        fails.append("spmmh_gemm brute force")
+    if not _close(Aa, ref_abs, ref_abs):
+        fails.append("spmmh_gemm magnitude companion")
+    if not np.all(A[1] == 0):
+        fails.append("spmmh_gemm empty row")
+    # D = 1: <SpMM,GEMM>, here by scipy's sparse product
+    Bs = sp.csr_matrix((vals.astype(np.float64), crd, pos), shape=(nrows, ncols))
+    A1, A1a = orc.spmmh_gemm(nrows, ncols, pos, crd, vals, C, np.ones_like(D), E)
+    if not _close(A1, (Bs @ C64) @ E64, A1a):
+        fails.append("spmmh_gemm D=1 is SpMM-GEMM")
+    # single nonzero B(i,k)=v: A[i,:] = v (C[k,:] * D[k,:]) . E
+    p1 = np.array([0, 0, 0, 0, 1], np.int32)
+    c1, v1 = np.array([6], np.int32), np.array([-1.25], np.float32)
+    As1, As1a = orc.spmmh_gemm(4, ncols, p1, c1, v1, C, D, E)
+    want = np.zeros((4, L)); want[3] = -1.25 * ((C64[6] * D64[6]) @ E64)
+    if not _close(As1, want, As1a):
+        fails.append("spmmh_gemm single nonzero")
+    # exact integers
+    pos_i, crd_i, vals_i = rand_csr(rng, 3, 5, 0.5, values="int")
+    Ci, Di, Ei = ints(rng, (5, 2)), ints(rng, (5, 2)), ints(rng, (2, 3))
+    Bi = csr_dense(3, 5, pos_i, crd_i, vals_i).astype(int).tolist()
+    Cl, Dl, El = (x.astype(int).tolist() for x in (Ci, Di, Ei))
+    exact = [[sum(Bi[i][k] * Cl[k][j] * Dl[k][j] * El[j][l] for k in range(5) for j in range(2)) for l in range(3)]
+             for i in range(3)]
+    Ae, _ = orc.spmmh_gemm(3, 5, pos_i, crd_i, vals_i, Ci, Di, Ei)
+    if not np.array_equal(Ae, np.array(exact, dtype=np.float64)):
+        fails.append("spmmh_gemm exact integers")
+    # linearity in C, D and E
+    Cy, C2 = dyadic(rng, (ncols, J)), dyadic(rng, (ncols, J))
+    Dy, D2 = dyadic(rng, (ncols, J)), dyadic(rng, (ncols, J))
+    Ey, E2 = dyadic(rng, (J, L)), dyadic(rng, (J, L))
+    a, b = 0.25, -3.0
+    run = lambda c, d, e: orc.spmmh_gemm(nrows, ncols, pos, crd, vals, c, d, e)
+    A0, s0 = run(Cy, Dy, Ey)
+    for name, args2, argsab in (("C", (C2, Dy, Ey), (combo(a, Cy, b, C2), Dy, Ey)),
+                                ("D", (Cy, D2, Ey), (Cy, combo(a, Dy, b, D2), Ey)),
+                                ("E", (Cy, Dy, E2), (Cy, Dy, combo(a, Ey, b, E2)))):
+        Aab, sab = run(*argsab)
+        A2, _ = run(*args2)
+        if not _close(Aab, a * A0 + b * A2, sab + s0):
+            fails.append(f"spmmh_gemm linear in {name}")
+    rows = np.array([5, 1, 2], np.int32)
+    As, _ = orc.spmmh_gemm(nrows, ncols, pos, crd, vals, C, D, E, rows=rows)
+    if not np.array_equal(As, A[rows]):
+        fails.append("spmmh_gemm row selection")
+    return fails
+
+
 ALL_CHECKS = {
     "spmm_gemm": check_spmm_gemm,
     "sddmm_spmm": check_sddmm_spmm,
     "mttkrp": check_mttkrp,
     "spttm_ttm": check_spttm_ttm,
+    "sddmm_spmm_gemm": check_sddmm_spmm_gemm,
+    "mttkrp_gemm": check_mttkrp_gemm,
+    "spmmh_gemm": check_spmmh_gemm,
 }
 
 

@@ -14,7 +14,7 @@ import _pins
 import oracle
 
 FUNCS = ["oracle_spmm_gemm(", "oracle_sddmm_spmm(", "oracle_mttkrp(", "oracle_spttm_ttm(",
-         "oracle_spttm_ttm_pattern("]
+         "oracle_spttm_ttm_pattern(", "oracle_sddmm_spmm_gemm(", "oracle_mttkrp_gemm(", "oracle_spmmh_gemm("]
 
 MUTANTS = [
     ("oracle_spmm_gemm(", "t[k] += b * c;", "t[k] += c;"),
@@ -37,6 +37,23 @@ MUTANTS = [
     ("oracle_spttm_ttm(", "t[l] += b * c;", "t[l] += b * b * c;"),
     ("oracle_spttm_ttm(", "A[s * M + m] = acc;", "A[s * M + m] = acc_abs;"),
     ("oracle_spttm_ttm_pattern(", "A_crd2[nf++] = crd2[f];", "A_crd2[nf++] = crd2[f] + (f == 0);"),
+    ("oracle_sddmm_spmm_gemm(", "y += b * c * d;", "y += c * d;"),
+    ("oracle_sddmm_spmm_gemm(", "t[l] += y * f;", "t[l] += f;"),
+    ("oracle_sddmm_spmm_gemm(", "W[(int64_t)l * M + m]", "W[(int64_t)m * L + l]"),
+    ("oracle_sddmm_spmm_gemm(", "C[(int64_t)i * K + k]", "C[(int64_t)(j % nrows) * K + k]"),
+    ("oracle_sddmm_spmm_gemm(", "t[l] = 0.0;", "(void)0;"),
+    ("oracle_sddmm_spmm_gemm(", "F[(int64_t)j * L + l]", "F[(int64_t)(i % ncols) * L + l]"),
+    ("oracle_mttkrp_gemm(", "u[l] += t[l] * c;", "u[l] = t[l] * c;"),
+    ("oracle_mttkrp_gemm(", "E[(int64_t)l * M + m]", "E[(int64_t)m * L + l]"),
+    ("oracle_mttkrp_gemm(", "t[l] += b * d;", "t[l] += d;"),
+    ("oracle_mttkrp_gemm(", "u[l] = 0.0;", "(void)0;"),
+    ("oracle_mttkrp_gemm(", "if (crd1[q] != i) continue;", "if (q != i) continue;"),
+    ("oracle_mttkrp_gemm(", "C[(int64_t)j * L + l]", "C[(int64_t)(i % d1) * L + l]"),
+    ("oracle_spmmh_gemm(", "t[j] += b * c * d;", "t[j] += b * c;"),
+    ("oracle_spmmh_gemm(", "t[j] += b * c * d;", "t[j] += b * c * c;"),
+    ("oracle_spmmh_gemm(", "E[(int64_t)j * L + l]", "E[(int64_t)l * J + j]"),
+    ("oracle_spmmh_gemm(", "acc += t[j] * e;", "acc -= t[j] * e;"),
+    ("oracle_spmmh_gemm(", "D[(int64_t)k * J + j]", "D[(int64_t)(k > 0 ? k - 1 : 0) * J + j]"),
 ]
 
 
