@@ -115,6 +115,12 @@ slnr_status slnr_sddmm_spmm_workspace(const slnr_csr *B, int32_t L, int32_t K, c
 slnr_status slnr_mttkrp_workspace(const slnr_csf3 *B, int32_t L, const slnr_opts *opts, size_t *bytes);
 slnr_status slnr_spttm_ttm_workspace(const slnr_csf3 *B, int32_t L, int32_t M, const slnr_opts *opts,
                                      size_t *bytes);
+slnr_status slnr_sddmm_spmm_gemm_workspace(const slnr_csr *B, int32_t K, int32_t L, int32_t M,
+                                           const slnr_opts *opts, size_t *bytes);
+slnr_status slnr_mttkrp_gemm_workspace(const slnr_csf3 *B, int32_t L, int32_t M, const slnr_opts *opts,
+                                       size_t *bytes);
+slnr_status slnr_spmmh_gemm_workspace(const slnr_csr *B, int32_t J, int32_t L, const slnr_opts *opts,
+                                      size_t *bytes);
 
 /* ---- <SpMM,GEMM>  (Sec. 6.2; case study Sec. 6.3) ----------------------
  * A(i,l) = sum_{j,k} B(i,j) * C(j,k) * D(k,l)
@@ -159,6 +165,41 @@ slnr_status slnr_mttkrp(const slnr_csf3 *B, const float *C, const float *D, int3
 slnr_status slnr_spttm_ttm(const slnr_csf3 *B, const float *C, int32_t L, const float *D, int32_t M,
                            int32_t *A_pos1, int32_t *A_crd1, int32_t *A_pos2, int32_t *A_crd2,
                            float *A_vals, const slnr_opts *opts);
+
+/* ---- <SDDMM,SpMM,GEMM>  (Sec. 6.2; recursive fusion, Sec. 4.2) ---------
+ * A(i,m) = sum_{j,k,l} B(i,j) * C(i,k) * D(j,k) * F(j,l) * W(l,m)
+ *   B: nrows x ncols CSR.  C: nrows x K.  D: ncols x K.  F: ncols x L.
+ *   W: L x M.  A: nrows x M (output).
+ * Fused: Algorithm 1 applied twice.  Per row i, per stored (i,j) the scalar
+ * y = B(i,j) C(i,:).D(j,:) is formed and T(i,:) += y F(j,:) at once; the row's
+ * vector temporary T(i,:) (length L) stays on chip and A(i,:) = T(i,:).W
+ * follows (fp32 FFMA).  Unfused: the sampled product Y (nnz values) and
+ * T = Y.F (nrows x L) are written to the workspace, then A = T.W (TF32 tensor
+ * cores with allow_tf32, where the widths allow). */
+slnr_status slnr_sddmm_spmm_gemm(const slnr_csr *B, const float *C, const float *D, int32_t K, const float *F,
+                                 int32_t L, const float *W, int32_t M, float *A, const slnr_opts *opts);
+
+/* ---- <MTTKRP,GEMM>  (Sec. 6.2) ------------------------------------------
+ * A(i,m) = sum_{j,k,l} B(i,j,k) * C(j,l) * D(k,l) * E(l,m)
+ *   B: d0 x d1 x d2 CSF.  C: d1 x L.  D: d2 x L.  E: L x M.  A: d0 x M (output).
+ *   (The paper writes the rank index as j: A_im = sum B_ikl C_lj D_kj E_jm.)
+ * Fused: as slnr_mttkrp, and each slice's MTTKRP row u(i,:) (length L) is
+ * formed on chip and multiplied by E at once (fp32 FFMA); rows without a
+ * slice are zero.  Unfused: the MTTKRP result (d0 x L) is written to the
+ * workspace (itself by the unfused MTTKRP schedule), then A = result.E. */
+slnr_status slnr_mttkrp_gemm(const slnr_csf3 *B, const float *C, const float *D, int32_t L, const float *E,
+                             int32_t M, float *A, const slnr_opts *opts);
+
+/* ---- <SpMMH,GEMM>  (Sec. 6.2) -------------------------------------------
+ * A(i,l) = sum_{k,j} B(i,k) * C(k,j) * D(k,j) * E(j,l)
+ *   B: nrows x ncols CSR.  C, D: ncols x J.  E: J x L.  A: nrows x L (output).
+ * Fused: per row i the temporary T(j) = sum_k B(i,k) C(k,j) D(k,j) (a sparse
+ * row times the Hadamard product of the gathered rows) is built on chip and
+ * multiplied by E at once, as in <SpMM,GEMM>.  Unfused: T (nrows x J) is
+ * written to the workspace, then A = T.E.  With allow_tf32 the T.E
+ * contraction may use TF32 tensor cores. */
+slnr_status slnr_spmmh_gemm(const slnr_csr *B, const float *C, const float *D, int32_t J, const float *E,
+                            int32_t L, float *A, const slnr_opts *opts);
 
 /* ---- <SDDMM,SpMM> without a caller workspace ----------------------------
  * The paper has no counterpart to this entry point; it serves callers that

@@ -60,10 +60,16 @@ SIGNATURES = {
     "slnr_sddmm_spmm_workspace": ([_CSR, _I32, _I32, _OPT, _SZ], ctypes.c_int),
     "slnr_mttkrp_workspace": ([_CSF, _I32, _OPT, _SZ], ctypes.c_int),
     "slnr_spttm_ttm_workspace": ([_CSF, _I32, _I32, _OPT, _SZ], ctypes.c_int),
+    "slnr_sddmm_spmm_gemm_workspace": ([_CSR, _I32, _I32, _I32, _OPT, _SZ], ctypes.c_int),
+    "slnr_mttkrp_gemm_workspace": ([_CSF, _I32, _I32, _OPT, _SZ], ctypes.c_int),
+    "slnr_spmmh_gemm_workspace": ([_CSR, _I32, _I32, _OPT, _SZ], ctypes.c_int),
     "slnr_spmm_gemm": ([_CSR, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_sddmm_spmm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_mttkrp": ([_CSF, _P, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_spttm_ttm": ([_CSF, _P, _I32, _P, _I32, _P, _P, _P, _P, _P, _OPT], ctypes.c_int),
+    "slnr_sddmm_spmm_gemm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
+    "slnr_mttkrp_gemm": ([_CSF, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
+    "slnr_spmmh_gemm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_sddmm_spmm_noalloc": ([_CSR, _P, _P, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
@@ -139,6 +145,18 @@ def slnr_mttkrp(B, C, D, L, A, opts):
 def slnr_spttm_ttm(B, C, L, D, M, A_pos1, A_crd1, A_pos2, A_crd2, A_vals, opts):
     return lib().slnr_spttm_ttm(ctypes.byref(B), C, L, D, M, A_pos1, A_crd1, A_pos2, A_crd2, A_vals,
                                 ctypes.byref(opts))
+
+
+def slnr_sddmm_spmm_gemm(B, C, D, K, F, L, W, M, A, opts):
+    return lib().slnr_sddmm_spmm_gemm(ctypes.byref(B), C, D, K, F, L, W, M, A, ctypes.byref(opts))
+
+
+def slnr_mttkrp_gemm(B, C, D, L, E, M, A, opts):
+    return lib().slnr_mttkrp_gemm(ctypes.byref(B), C, D, L, E, M, A, ctypes.byref(opts))
+
+
+def slnr_spmmh_gemm(B, C, D, J, E, L, A, opts):
+    return lib().slnr_spmmh_gemm(ctypes.byref(B), C, D, J, E, L, A, ctypes.byref(opts))
 
 
 def _query(fn_name, *args):
@@ -351,6 +369,57 @@ def spttm_ttm(B: DeviceCSF3, C, D, out=None, variant="fused", allow_tf32=True, v
     return p1, c1[:B.nslices], p2, c2[:B.nfibers], v
 
 
+def sddmm_spmm_gemm(B: DeviceCSR, C, D, F, W, out=None, variant="fused", allow_tf32=True, validate=False,
+                    workspace=None, stream=None):
+    """A(i,m) = sum_{j,k,l} B(i,j) C(i,k) D(j,k) F(j,l) W(l,m)  (<SDDMM,SpMM,GEMM>, Sec. 6.2)."""
+    torch = _torch()
+    C, D, F, W = _dense(C, "C"), _dense(D, "D"), _dense(F, "F"), _dense(W, "W")
+    K, L, M = C.shape[1], F.shape[1], W.shape[1]
+    if out is None:
+        out = torch.empty((B.nrows, M), dtype=torch.float32, device=C.device)
+    o = _opts(variant, allow_tf32, validate, stream)
+    bs = B.c_struct()
+    n = _query("slnr_sddmm_spmm_gemm_workspace", ctypes.byref(bs), K, L, M, ctypes.byref(o))
+    _keep = _attach_ws(o, n, workspace)
+    _check(slnr_sddmm_spmm_gemm(bs, C.data_ptr(), D.data_ptr(), K, F.data_ptr(), L, W.data_ptr(), M,
+                                out.data_ptr(), o), "slnr_sddmm_spmm_gemm")
+    return out
+
+
+def mttkrp_gemm(B: DeviceCSF3, C, D, E, out=None, variant="fused", allow_tf32=True, validate=False, workspace=None,
+                stream=None):
+    """A(i,m) = sum_{j,k,l} B(i,j,k) C(j,l) D(k,l) E(l,m)  (<MTTKRP,GEMM>, Sec. 6.2)."""
+    torch = _torch()
+    C, D, E = _dense(C, "C"), _dense(D, "D"), _dense(E, "E")
+    L, M = C.shape[1], E.shape[1]
+    if out is None:
+        out = torch.empty((B.dims[0], M), dtype=torch.float32, device=C.device)
+    o = _opts(variant, allow_tf32, validate, stream)
+    bs = B.c_struct()
+    n = _query("slnr_mttkrp_gemm_workspace", ctypes.byref(bs), L, M, ctypes.byref(o))
+    _keep = _attach_ws(o, n, workspace)
+    _check(slnr_mttkrp_gemm(bs, C.data_ptr(), D.data_ptr(), L, E.data_ptr(), M, out.data_ptr(), o),
+           "slnr_mttkrp_gemm")
+    return out
+
+
+def spmmh_gemm(B: DeviceCSR, C, D, E, out=None, variant="fused", allow_tf32=True, validate=False, workspace=None,
+               stream=None):
+    """A(i,l) = sum_{k,j} B(i,k) C(k,j) D(k,j) E(j,l)  (<SpMMH,GEMM>, Sec. 6.2)."""
+    torch = _torch()
+    C, D, E = _dense(C, "C"), _dense(D, "D"), _dense(E, "E")
+    J, L = C.shape[1], E.shape[1]
+    if out is None:
+        out = torch.empty((B.nrows, L), dtype=torch.float32, device=C.device)
+    o = _opts(variant, allow_tf32, validate, stream)
+    bs = B.c_struct()
+    n = _query("slnr_spmmh_gemm_workspace", ctypes.byref(bs), J, L, ctypes.byref(o))
+    _keep = _attach_ws(o, n, workspace)
+    _check(slnr_spmmh_gemm(bs, C.data_ptr(), D.data_ptr(), J, E.data_ptr(), L, out.data_ptr(), o),
+           "slnr_spmmh_gemm")
+    return out
+
+
 def run(op: str, B, dense: dict, **kw):
     """Dispatch by operation name with the dense operands of a workload."""
     if op == "spmm_gemm":
@@ -361,4 +430,10 @@ def run(op: str, B, dense: dict, **kw):
         return mttkrp(B, dense["C"], dense["D"], **kw)
     if op == "spttm_ttm":
         return spttm_ttm(B, dense["C"], dense["D"], **kw)
+    if op == "sddmm_spmm_gemm":
+        return sddmm_spmm_gemm(B, dense["C"], dense["D"], dense["F"], dense["W"], **kw)
+    if op == "mttkrp_gemm":
+        return mttkrp_gemm(B, dense["C"], dense["D"], dense["E"], **kw)
+    if op == "spmmh_gemm":
+        return spmmh_gemm(B, dense["C"], dense["D"], dense["E"], **kw)
     raise ValueError(op)

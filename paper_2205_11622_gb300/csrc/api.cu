@@ -107,8 +107,9 @@ struct Layout {
     o_heavy = take(sizeof(HeavyRow) * (size_t)mh);
     o_partial = take(sizeof(float) * (size_t)mc * (size_t)width);
   }
-  size_t o_inter = 0;
+  size_t o_inter = 0, o_inter2 = 0;
   void inter(size_t bytes) { o_inter = take(bytes); }
+  void inter2(size_t bytes) { o_inter2 = take(bytes); }
   size_t total() const { return align256(cur); }
 };
 
@@ -270,6 +271,27 @@ Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opt
   return l;
 }
 
+Layout layout_sddmm_spmm_gemm(const slnr_csr* B, int32_t L, int variant) {
+  Layout l;
+  l.split(B->nrows, B->nnz, L);
+  if (variant == SLNR_UNFUSED) {
+    l.inter(sizeof(float) * (size_t)B->nnz);                      // Y
+    l.inter2(sizeof(float) * (size_t)B->nrows * (size_t)L);       // T = Y.F
+  }
+  return l;
+}
+
+Layout layout_mttkrp_gemm(const slnr_csf3* B, int32_t L, int variant) {
+  Layout l;
+  l.units(B->nslices, B->nnz, L);
+  if (variant == SLNR_UNFUSED) {
+    l.split(B->nfibers, B->nnz, L);
+    l.inter(sizeof(float) * (size_t)B->nfibers * (size_t)L);      // per-fiber T
+    l.inter2(sizeof(float) * (size_t)B->dim[0] * (size_t)L);      // the MTTKRP result
+  }
+  return l;
+}
+
 CsrView csr_view(const slnr_csr* B) { return CsrView{B->nrows, B->ncols, B->nnz, B->pos, B->crd, B->vals}; }
 CsrView fiber_view(const slnr_csf3* B) {
   return CsrView{B->nfibers, B->dim[2], B->nnz, B->pos3, B->crd3, B->vals};
@@ -361,6 +383,40 @@ slnr_status slnr_spttm_ttm_workspace(const slnr_csf3* B, int32_t L, int32_t M, c
   SLNR_CHECK(check_dims("M", M));
   if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
   *bytes = layout_spttm_ttm(B, L, M, opts).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_sddmm_spmm_gemm_workspace(const slnr_csr* B, int32_t K, int32_t L, int32_t M, const slnr_opts* opts,
+                                           size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, false));
+  SLNR_CHECK(check_dims("K", K));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_sddmm_spmm_gemm(B, L, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_mttkrp_gemm_workspace(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opts* opts,
+                                       size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, false));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_mttkrp_gemm(B, L, opts->variant).total();
+  return SLNR_OK;
+}
+
+slnr_status slnr_spmmh_gemm_workspace(const slnr_csr* B, int32_t J, int32_t L, const slnr_opts* opts,
+                                      size_t* bytes) {
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, false));
+  SLNR_CHECK(check_dims("J", J));
+  SLNR_CHECK(check_dims("L", L));
+  if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
+  *bytes = layout_spmm_gemm(B, J, L, opts).total();
   return SLNR_OK;
 }
 
@@ -482,7 +538,7 @@ slnr_status slnr_mttkrp(const slnr_csf3* B, const float* C, const float* D, int3
     SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
     SLNR_LAUNCH("mttkrp_stage2_units", launch_mttkrp_stage2_units(L, *B, T, C, up, s));
   }
-  SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, A, s));
+  SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, nullptr, 0, A, s));
   timing_end(s);
   return SLNR_OK;
 }
@@ -539,6 +595,147 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
         SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nfibers, L, M, T, D, A_vals, sp.hdr, s));
       else
         SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nfibers, L, M, T, D, A_vals, 0, s));
+    }
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float* D, int32_t K, const float* F,
+                                 int32_t L, const float* W, int32_t M, float* A, const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, true));
+  SLNR_CHECK(check_dims("K", K));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("F", F));
+  SLNR_CHECK(check_dense("W", W));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_sddmm_spmm_gemm(B, L, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->nrows == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
+  const CsrView v = csr_view(B);
+  const SplitPlan sp = split_plan(ws, l);
+  SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+  if (opts->variant == SLNR_FUSED) {
+    // heavy rows: partial T rows (width L), then their fixed-order sum times W
+    SLNR_LAUNCH("sddmm_spmm_chunks", launch_sddmm_spmm_chunks(v, C, D, K, F, L, sp, s));
+    SLNR_LAUNCH("sddmm_spmm_gemm_tiles", launch_sddmm_spmm_gemm_tiles(v, C, D, K, F, L, W, M, A, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, W, M, A, s));
+  } else {
+    float* Y = reinterpret_cast<float*>(ws + l.o_inter);
+    float* T = reinterpret_cast<float*>(ws + l.o_inter2);
+    SLNR_LAUNCH("sddmm_rows", launch_sddmm_rows(v, C, D, K, Y, s));
+    SLNR_LAUNCH("sddmm_chunks", launch_sddmm_chunks(v, C, D, K, Y, sp, s));
+    CsrView vy = v;
+    vy.vals = Y;
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, vy, F, sp, s));
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, vy, F, T, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
+    if (use_tc(opts, L, M))
+      SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nrows, L, M, T, W, A, sp.hdr, s));
+    else
+      SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, L, M, T, W, A, 0, s));
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_mttkrp_gemm(const slnr_csf3* B, const float* C, const float* D, int32_t L, const float* E,
+                             int32_t M, float* A, const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csf(B, true));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dims("M", M));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("E", E));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_mttkrp_gemm(B, L, opts->variant);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->dim[0] == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
+  const UnitPlan up = unit_plan(ws, l);
+  SLNR_LAUNCH("csf_units", launch_csf_units(*B, up, s));
+  if (opts->variant == SLNR_FUSED) {
+    SLNR_LAUNCH("mttkrp_units", launch_mttkrp_units(L, *B, C, D, up, s));
+    SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, E, M, A, s));
+  } else {
+    const CsrView fv = fiber_view(B);
+    const SplitPlan sp = split_plan(ws, l);
+    float* T = reinterpret_cast<float*>(ws + l.o_inter);
+    float* U = reinterpret_cast<float*>(ws + l.o_inter2);
+    SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(L, fv, D, sp, s));
+    SLNR_LAUNCH("spmm_rows", launch_spmm_rows(L, fv, D, T, s));
+    SLNR_LAUNCH("combine", launch_combine(L, sp, nullptr, 0, T, s));
+    SLNR_LAUNCH("mttkrp_stage2_units", launch_mttkrp_stage2_units(L, *B, T, C, up, s));
+    SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, nullptr, 0, U, s));
+    if (use_tc(opts, L, M))
+      SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->dim[0], L, M, U, E, A, sp.hdr, s));
+    else
+      SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->dim[0], L, M, U, E, A, 0, s));
+  }
+  timing_end(s);
+  return SLNR_OK;
+}
+
+slnr_status slnr_spmmh_gemm(const slnr_csr* B, const float* C, const float* D, int32_t J, const float* E,
+                            int32_t L, float* A, const slnr_opts* opts) {
+  g_last_error[0] = '\0';
+  timing_begin();
+  SLNR_CHECK(check_opts(opts));
+  SLNR_CHECK(check_csr(B, true));
+  SLNR_CHECK(check_dims("J", J));
+  SLNR_CHECK(check_dims("L", L));
+  SLNR_CHECK(check_dense("C", C));
+  SLNR_CHECK(check_dense("D", D));
+  SLNR_CHECK(check_dense("E", E));
+  SLNR_CHECK(check_dense("A", A));
+  const Layout l = layout_spmm_gemm(B, J, L, opts);
+  SLNR_CHECK(check_ws(opts, l.total()));
+  if (B->nrows == 0) return SLNR_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
+  char* ws = static_cast<char*>(opts->workspace);
+  SLNR_CHECK(begin(ws, s, opts->validate != 0,
+                   [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
+  const CsrView v = csr_view(B);
+  const bool tc = use_tc(opts, J, L);
+  // the gathered row of column k is C(k,:) .* D(k,:); E is the consumer matrix
+  if (opts->variant == SLNR_FUSED && tc) {
+    const SegPlan gp = seg_plan(ws, l);
+    SLNR_LAUNCH("seg_count", launch_seg_count(v, gp, s));
+    SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
+    SLNR_LAUNCH("tc_spmmh_gemm", launch_tc_spmm_gemm(J, L, v, C, E, A, gp, s, D));
+    SLNR_LAUNCH("combine", launch_combine(L, combine_plan(gp), nullptr, 0, A, s));
+  } else {
+    const SplitPlan sp = split_plan(ws, l);
+    SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+    SLNR_LAUNCH("spmm_chunks", launch_spmm_chunks(J, v, C, sp, s, D));
+    if (opts->variant == SLNR_FUSED) {
+      SLNR_LAUNCH("spmm_gemm_tiles", launch_spmm_gemm_tiles(J, L, v, C, E, A, 0, s, D));
+      SLNR_LAUNCH("combine", launch_combine(J, sp, E, L, A, s));
+    } else {
+      float* T = reinterpret_cast<float*>(ws + l.o_inter);
+      SLNR_LAUNCH("spmm_rows", launch_spmm_rows(J, v, C, T, s, D));
+      SLNR_LAUNCH("combine", launch_combine(J, sp, nullptr, 0, T, s));
+      if (tc)
+        SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nrows, J, L, T, E, A, sp.hdr, s));
+      else
+        SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, J, L, T, E, A, 0, s));
     }
   }
   timing_end(s);

@@ -129,11 +129,14 @@ __device__ __forceinline__ void zero_vec(float (&v)[VPL]) {
 
 // acc += sum_{p in [p0,p1)} vals[p] * X[crd[p], col .. col+VPL)
 // Sequential in p for every element (fixed order).  U independent row loads
-// are in flight per step.
-template <int VPL, int U = 4>
+// are in flight per step.  With H (the Hadamard gather of <SpMMH,GEMM>) the
+// gathered row is X[crd[p], :] .* X2[crd[p], :], the product formed in fp32
+// before the multiply-add.
+template <int VPL, int U = 4, bool H = false>
 __device__ __forceinline__ void gather_acc(float (&acc)[VPL], const int32_t* __restrict__ crd,
                                            const float* __restrict__ vals, int p0, int p1,
-                                           const float* __restrict__ X, int ldx, int col) {
+                                           const float* __restrict__ X, int ldx, int col,
+                                           const float* __restrict__ X2 = nullptr) {
   int p = p0;
   for (; p + U <= p1; p += U) {
     int c[U];
@@ -146,6 +149,15 @@ __device__ __forceinline__ void gather_acc(float (&acc)[VPL], const int32_t* __r
     float x[U][VPL];
 #pragma unroll
     for (int u = 0; u < U; ++u) ldg_vec<VPL>(x[u], X + (int64_t)c[u] * ldx + col);
+    if constexpr (H) {
+      float x2[U][VPL];
+#pragma unroll
+      for (int u = 0; u < U; ++u) ldg_vec<VPL>(x2[u], X2 + (int64_t)c[u] * ldx + col);
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int e = 0; e < VPL; ++e) x[u][e] *= x2[u][e];
+    }
 #pragma unroll
     for (int u = 0; u < U; ++u)
 #pragma unroll
@@ -156,6 +168,12 @@ __device__ __forceinline__ void gather_acc(float (&acc)[VPL], const int32_t* __r
     const float v = __ldg(vals + p);
     float x[VPL];
     ldg_vec<VPL>(x, X + (int64_t)c * ldx + col);
+    if constexpr (H) {
+      float x2[VPL];
+      ldg_vec<VPL>(x2, X2 + (int64_t)c * ldx + col);
+#pragma unroll
+      for (int e = 0; e < VPL; ++e) x[e] *= x2[e];
+    }
 #pragma unroll
     for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v, x[e], acc[e]);
   }

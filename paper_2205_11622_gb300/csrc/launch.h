@@ -66,9 +66,11 @@ cudaError_t launch_validate_csr(const slnr_csr& B, WsHeader* hdr, cudaStream_t s
 cudaError_t launch_validate_csf(const slnr_csf3& B, WsHeader* hdr, cudaStream_t s);
 
 // spmm.cu -- out[r,:] = sum_p vals[p] X[crd[p],:] (width W), and the heavy-row machinery
-cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s);
+// (with X2 not NULL the gathered row is X[k,:] .* X2[k,:], the <SpMMH,GEMM> producer)
+cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s,
+                             const float* X2 = nullptr);
 cudaError_t launch_spmm_chunks(int W, const CsrView& B, const float* X, const SplitPlan& plan,
-                               cudaStream_t s);
+                               cudaStream_t s, const float* X2 = nullptr);
 // heavy rows: out[row,:] = sum of the row's partials (width W); when D is not
 // NULL the sum (width W = K) is multiplied by D (K x L) and out has width L.
 cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, float* out,
@@ -76,7 +78,7 @@ cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, 
 
 // gemm.cu -- fused SpMM x D over light rows; dense GEMM for the unfused variant
 cudaError_t launch_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* C, const float* D,
-                                   float* A, int use_tf32, cudaStream_t s);
+                                   float* A, int use_tf32, cudaStream_t s, const float* C2 = nullptr);
 cudaError_t launch_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                               int use_tf32, cudaStream_t s);
 
@@ -85,8 +87,9 @@ bool tc_supported(int K, int L);
 int seg_scan_blocks(int64_t nrows);
 cudaError_t launch_seg_count(const CsrView& B, const SegPlan& plan, cudaStream_t s);
 cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t s);
+// (with C2 not NULL the gathered row is C[k,:] .* C2[k,:], <SpMMH,GEMM>)
 cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, const float* D, float* A,
-                                const SegPlan& plan, cudaStream_t s);
+                                const SegPlan& plan, cudaStream_t s, const float* C2 = nullptr);
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s);
 
@@ -95,6 +98,9 @@ cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float
                                    const float* E, int K, float* A, cudaStream_t s);
 cudaError_t launch_sddmm_spmm_chunks(const CsrView& B, const float* C, const float* D, int L,
                                      const float* E, int K, const SplitPlan& plan, cudaStream_t s);
+// fused <SDDMM,SpMM,GEMM> over light rows: C nrows x K, D ncols x K, F ncols x L, W L x M
+cudaError_t launch_sddmm_spmm_gemm_tiles(const CsrView& B, const float* C, const float* D, int K,
+                                         const float* F, int L, const float* W, int M, float* A, cudaStream_t s);
 cudaError_t launch_sddmm_rows(const CsrView& B, const float* C, const float* D, int L, float* Y,
                               cudaStream_t s);
 cudaError_t launch_sddmm_chunks(const CsrView& B, const float* C, const float* D, int L, float* Y,
@@ -105,8 +111,10 @@ cudaError_t launch_mttkrp_units(int L, const slnr_csf3& B, const float* C, const
                                 const UnitPlan& plan, cudaStream_t s);
 cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T, const float* C,
                                        const UnitPlan& plan, cudaStream_t s);
-cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, float* A,
-                                  cudaStream_t s);
+// A(i,:) = sum of slice i's unit partials (width L); with E (L x M) not NULL,
+// that sum times E (A has width M).
+cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M,
+                                  float* A, cudaStream_t s);
 
 }  // namespace slnr
 

@@ -1,4 +1,5 @@
 // MTTKRP:  A(i,l) = sum_{j,k} B(i,j,k) * C(j,l) * D(k,l),  B in CSF (i -> j -> k)
+// and <MTTKRP,GEMM>: the same followed by A(i,:).E.
 //
 // Fused schedule (Sec. 4.2, Algorithm 1 removing C): the shared loops are the
 // slice i and the fiber j; the producer builds T(l) = sum_k B(i,j,k) D(k,l)
@@ -112,10 +113,14 @@ __global__ void __launch_bounds__(256) k_mttkrp_stage2_units(const WsHeader* __r
 
 // One CTA per output row i: find i's slice, sum its units' partials (strided
 // lanes, then a fixed pairwise tree), write A(i,:) (zeros without a slice).
+// With E (L x M, <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and
+// A(i,:) = u(i,:).E is written instead (width M): the MTTKRP result is never
+// stored.
 template <int L>
 __global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, const int32_t* __restrict__ crd1,
                                                         const SliceUnits* __restrict__ sus,
                                                         const float* __restrict__ partial,
+                                                        const float* __restrict__ E, int M,
                                                         float* __restrict__ A) {
   constexpr int NC = L / 4;
   constexpr int NR = 256 / NC;
@@ -149,7 +154,17 @@ __global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, con
       }
       __syncthreads();
     }
-    if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
+    if (E == nullptr) {
+      if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
+    } else {
+      const float* u = reinterpret_cast<const float*>(red);  // u(i,0..L)
+      for (int m = threadIdx.x; m < M; m += blockDim.x) {
+        float acc = 0.f;
+#pragma unroll 8
+        for (int l = 0; l < L; ++l) acc = fmaf(u[l], __ldg(E + (int64_t)l * M + m), acc);
+        A[(int64_t)i * M + m] = acc;
+      }
+    }
     __syncthreads();
   }
 }
@@ -184,14 +199,15 @@ cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T
   return cudaGetLastError();
 }
 
-cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, float* A,
-                                  cudaStream_t s) {
+cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M,
+                                  float* A, cudaStream_t s) {
   if (B.dim[0] <= 0) return cudaSuccess;
   int grid = B.dim[0];
   const int cap = device_sm_count() * 8;
   if (grid > cap) grid = cap;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.dim[0], B.nslices, B.crd1, plan.slice_units, plan.partial, A);
+    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.dim[0], B.nslices, B.crd1, plan.slice_units, plan.partial, E, M,
+                                              A);
   });
   return cudaGetLastError();
 }

@@ -12,6 +12,7 @@
 // Unfused schedule (Fig. 2a then Fig. 2b): Y(i,j) for every stored (i,j) is
 // written to memory, then A = Y.E runs as an SpMM (spmm.cu).
 #include "launch.h"
+#include "tile.cuh"
 
 namespace slnr {
 namespace {
@@ -110,6 +111,54 @@ __global__ void __launch_bounds__(256) k_sddmm_spmm_chunks(const WsHeader* __res
   }
 }
 
+// Fused <SDDMM,SpMM,GEMM> over light rows (Algorithm 1 applied twice): a CTA
+// owns kTileRows consecutive rows; a warp builds a row's temporary
+// T(i,:) = sum_j B(i,j) <C(i,:), D(j,:)> F(j,:) (scalar per nonzero, vector
+// of width LW per row) into the shared-memory tile, then the tile is
+// multiplied by W (LW x M) and A's rows are written once.  Rows with more than
+// kLightMax nonzeros are left to the chunk kernel and k_combine (times W).
+template <int WM, int LW>
+__global__ void __launch_bounds__(256) k_sddmm_spmm_gemm_tiles(int nrows, const int32_t* __restrict__ pos,
+                                                               const int32_t* __restrict__ crd,
+                                                               const float* __restrict__ vals,
+                                                               const float* __restrict__ C,
+                                                               const float* __restrict__ D, int K,
+                                                               const float* __restrict__ F,
+                                                               const float* __restrict__ W, int M,
+                                                               float* __restrict__ A) {
+  using RL = RowLanes<WM>;
+  extern __shared__ float4 smem4[];
+  float* T = reinterpret_cast<float*>(smem4);
+  float* Ws = T + kTileRows * LW;
+  __shared__ int keep[kTileRows];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t r0 = (int64_t)blockIdx.x * kTileRows;
+  for (int rr = warp; rr < kTileRows; rr += 8) {
+    const int64_t r = r0 + rr;
+    float c[RL::VPL], acc[RL::VPL];
+    zero_vec(acc);
+    int ok = 0;
+    if (r < nrows) {
+      const int p0 = pos[r], p1 = pos[r + 1];
+      if (p1 - p0 <= kLightMax) {  // warp-uniform
+        if (col < K) ldg_vec_upto<RL::VPL>(c, C + r * K + col, K - col); else zero_vec(c);
+        sddmm_spmm_range<WM>(acc, c, p0, p1, crd, vals, D, K, F, LW, grp, col);
+        cross_group_sum<RL::GS>(acc);
+        ok = 1;
+      }
+    }
+    if (grp == 0 && col < LW) {
+#pragma unroll
+      for (int x = 0; x < RL::VPL; ++x)
+        if (col + x < LW) T[rr * LW + col + x] = acc[x];
+    }
+    if (lane == 0) keep[rr] = ok;
+  }
+  __syncthreads();
+  tile_times_d<LW>(T, W, M, Ws, A, r0, nrows, keep);
+}
+
 // Unfused producer: Y[p] = vals[p] * <C(i,:), D(crd[p],:)> for p in [p0, p1) of row i.
 template <int W>
 __device__ __forceinline__ void sddmm_range(const float (&c)[RowLanes<W>::VPL], int p0, int p1,
@@ -197,6 +246,25 @@ cudaError_t launch_sddmm_spmm_chunks(const CsrView& B, const float* C, const flo
     k_sddmm_spmm_chunks<W><<<grid_rows(plan.max_chunks), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks,
                                                                       B.crd, B.vals, C, D, L, E, K,
                                                                       plan.partial);
+  });
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sddmm_spmm_gemm_tiles(const CsrView& B, const float* C, const float* D, int K,
+                                         const float* F, int L, const float* W, int M, float* A, cudaStream_t s) {
+  if (B.nrows <= 0) return cudaSuccess;
+  const int64_t grid = ceil_div(B.nrows, kTileRows);
+  const size_t smem = tile_smem_bytes(L, M);
+  const int WM = K > L ? K : L;
+  SLNR_WIDTH_SWITCH(WM, WMC, {
+    SLNR_WIDTH_SWITCH(L, LC, {
+      if (LC <= WMC) {
+        cudaError_t e = set_smem(k_sddmm_spmm_gemm_tiles<WMC, LC <= WMC ? LC : WMC>, smem);
+        if (e != cudaSuccess) return e;
+        k_sddmm_spmm_gemm_tiles<WMC, LC <= WMC ? LC : WMC><<<(unsigned)grid, 256, smem, s>>>(
+            B.nrows, B.pos, B.crd, B.vals, C, D, K, F, W, M, A);
+      }
+    });
   });
   return cudaGetLastError();
 }

@@ -5,17 +5,19 @@
 // This is the SpMM of Fig. 2b and the producer of <SpMM,GEMM> (T = B.C),
 // of <SpTTM,SpTTM> (T = B x_3 C per fiber) and of MTTKRP's unfused variant.
 // A group of lanes owns one row (common.cuh, RowLanes), so light rows need no
-// cross-lane reduction; heavy rows go through chunks and k_combine.
+// cross-lane reduction; heavy rows go through chunks and k_combine.  With H
+// the gathered row is X[k,:] .* X2[k,:] (the producer of <SpMMH,GEMM>).
 #include "launch.h"
 
 namespace slnr {
 namespace {
 
-template <int W>
+template <int W, bool H>
 __global__ void __launch_bounds__(256) k_spmm_rows(int nrows, const int32_t* __restrict__ pos,
                                                    const int32_t* __restrict__ crd,
                                                    const float* __restrict__ vals,
-                                                   const float* __restrict__ X, float* __restrict__ out) {
+                                                   const float* __restrict__ X, const float* __restrict__ X2,
+                                                   float* __restrict__ out) {
   using RL = RowLanes<W>;
   const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -25,17 +27,17 @@ __global__ void __launch_bounds__(256) k_spmm_rows(int nrows, const int32_t* __r
     if (p1 - p0 > kLightMax) continue;  // written by the heavy-row path
     float acc[RL::VPL];
     zero_vec(acc);
-    gather_acc<RL::VPL>(acc, crd, vals, p0, p1, X, W, col);
+    gather_acc<RL::VPL, H ? 2 : 4, H>(acc, crd, vals, p0, p1, X, W, col, X2);
     st_vec(out + r * W + col, acc);
   }
 }
 
-template <int W>
+template <int W, bool H>
 __global__ void __launch_bounds__(256) k_spmm_chunks(const WsHeader* __restrict__ hdr,
                                                      const Chunk* __restrict__ chunks, int max_chunks,
                                                      const int32_t* __restrict__ crd,
                                                      const float* __restrict__ vals,
-                                                     const float* __restrict__ X,
+                                                     const float* __restrict__ X, const float* __restrict__ X2,
                                                      float* __restrict__ partial) {
   using RL = RowLanes<W>;
   const int n = min(hdr->n_chunks, max_chunks);
@@ -46,7 +48,7 @@ __global__ void __launch_bounds__(256) k_spmm_chunks(const WsHeader* __restrict_
     const Chunk ch = chunks[c];
     float acc[RL::VPL];
     zero_vec(acc);
-    gather_acc<RL::VPL>(acc, crd, vals, ch.p0, ch.p1, X, W, col);
+    gather_acc<RL::VPL, H ? 2 : 4, H>(acc, crd, vals, ch.p0, ch.p1, X, W, col, X2);
     st_vec(partial + (int64_t)ch.slot * W + col, acc);
   }
 }
@@ -119,20 +121,30 @@ inline int grid_warps(int64_t items_per_warp_round, int64_t n) {
 
 }  // namespace
 
-cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s) {
+cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out, cudaStream_t s,
+                             const float* X2) {
   if (B.nrows <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(W, WC, {
-    k_spmm_rows<WC><<<grid_warps(RowLanes<WC>::GPW, B.nrows), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, out);
+    const int grid = grid_warps(RowLanes<WC>::GPW, B.nrows);
+    if (X2 == nullptr)
+      k_spmm_rows<WC, false><<<grid, 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, nullptr, out);
+    else
+      k_spmm_rows<WC, true><<<grid, 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, X2, out);
   });
   return cudaGetLastError();
 }
 
 cudaError_t launch_spmm_chunks(int W, const CsrView& B, const float* X, const SplitPlan& plan,
-                               cudaStream_t s) {
+                               cudaStream_t s, const float* X2) {
   if (plan.max_chunks <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(W, WC, {
-    k_spmm_chunks<WC><<<grid_warps(RowLanes<WC>::GPW, plan.max_chunks), 256, 0, s>>>(
-        plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X, plan.partial);
+    const int grid = grid_warps(RowLanes<WC>::GPW, plan.max_chunks);
+    if (X2 == nullptr)
+      k_spmm_chunks<WC, false><<<grid, 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X,
+                                                     nullptr, plan.partial);
+    else
+      k_spmm_chunks<WC, true><<<grid, 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X, X2,
+                                                    plan.partial);
   });
   return cudaGetLastError();
 }

@@ -18,7 +18,8 @@
 // order: A(r,:) = sum_chunks T_chunk . D, which is exact by linearity.
 //
 // The same kernel in DENSE mode multiplies a materialised T (unfused
-// variant) by D: the producer reads T rows instead of gathering them.
+// variant) by D: the producer reads T rows instead of gathering them.  In
+// Hadamard mode (<SpMMH,GEMM>) the gathered row is C(k,:) .* C2(k,:).
 #include "launch.h"
 #include "tcgen05.cuh"
 
@@ -176,7 +177,9 @@ __device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity
   return true;
 }
 
-enum TcMode { kSegments = 0, kDense = 1 };
+// kSegments: gathered row segments; kSegmentsH: the same with Hadamard rows
+// X[k,:] .* X2[k,:] (<SpMMH,GEMM>); kDense: rows of a materialised T.
+enum TcMode { kSegments = 0, kDense = 1, kSegmentsH = 2 };
 
 // Number of T / accumulator buffers: up to four, as many as fit beside D^T
 // in shared memory (200 KB budget) and in tensor memory (512 columns).
@@ -252,7 +255,8 @@ template <int K, int L, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_gemm(WsHeader* hdr, const int4* __restrict__ segs, int max_segs,
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
-              const float* __restrict__ X, const float* __restrict__ D, float* __restrict__ A,
+              const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ D,
+              float* __restrict__ A,
               float* __restrict__ partial) {
   static_assert(K % 32 == 0 && K >= 32 && K <= 128, "K must be 32, 64 or 128");
   static_assert(L % 32 == 0 && L >= 32 && L <= 256, "L must be a multiple of 32 in [32, 256]");
@@ -278,7 +282,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   if (tid == 0) {
     for (int b = 0; b < NBUF; ++b) {
-      tc::mbar_init(&full_bar[b], kTcRows / (PL::G * (MODE == kSegments ? 1 : SLNR_TC_DENSE_ROWS)));  // one arrival per claim
+      tc::mbar_init(&full_bar[b], kTcRows / (PL::G * (MODE != kDense ? 1 : SLNR_TC_DENSE_ROWS)));  // one arrival per claim
       tc::mbar_init(&mma_bar[b], 1);
       tc::mbar_init(&free_bar[b], 4);
       last_commit[b] = -1;
@@ -304,7 +308,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t tmem = tmem_base;
 
   int64_t nitems;
-  if (MODE == kSegments) {
+  if (MODE != kDense) {
     const int n = hdr->n_segs;
     nitems = n < max_segs ? n : max_segs;
   } else {
@@ -323,7 +327,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // then waits for its buffer to be free (the MMAs of tile c / CPT - NBUF
     // completed and their destinations read), stores the rows and their
     // destinations, and lane 0 arrives once for the claim.
-    constexpr int VPL = PL::VPL, G = PL::G, R = MODE == kSegments ? 1 : SLNR_TC_DENSE_ROWS;
+    constexpr int VPL = PL::VPL, G = PL::G, R = MODE != kDense ? 1 : SLNR_TC_DENSE_ROWS;
     constexpr int IPC = G * R, CPT = kTcRows / IPC;
     static_assert(kTcRows % IPC == 0, "claims tile the item tile");
     const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
@@ -333,7 +337,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (c < nclaims) {
         const int64_t item =
             ((int64_t)blockIdx.x + (int64_t)(c / CPT) * gridDim.x) * kTcRows + (c % CPT) * IPC + r * G + g;
-        if (item < nitems) rv = (MODE == kSegments) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
+        if (item < nitems) rv = (MODE != kDense) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
       }
       return rv;
     };
@@ -347,10 +351,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int cl_next = __shfl_sync(0xffffffffu, x, 0);
       float acc[R][VPL];
       int2 dst0 = make_int2(-1, -1);  // destination of the segment (R = 1)
-      if constexpr (MODE == kSegments) {
+      if constexpr (MODE != kDense) {
         const int4 rec_next = load_rec(cl_next, 0);  // loads while this claim is built
         zero_vec(acc[0]);
-        if (rec.x >= 0) gather_acc<VPL, PL::U>(acc[0], crd, vals, rec.y, rec.z, X, K, col);
+        if (rec.x >= 0) {
+          if constexpr (MODE == kSegmentsH)
+            gather_acc<VPL, PL::U / 2, true>(acc[0], crd, vals, rec.y, rec.z, X, K, col, X2);
+          else
+            gather_acc<VPL, PL::U>(acc[0], crd, vals, rec.y, rec.z, X, K, col);
+        }
         dst0 = make_int2(rec.x, rec.w);
         rec = rec_next;
       } else {
@@ -373,7 +382,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int r = 0; r < R; ++r) {
         store_t_part<VPL>(sT + b * TBYTES, s0 + r * G, col, acc[r]);
         if (lane % PL::GS == 0)
-          dest[b][s0 + r * G] = MODE == kSegments ? dst0 : make_int2(load_rec(cl, r).x, -1);
+          dest[b][s0 + r * G] = MODE != kDense ? dst0 : make_int2(load_rec(cl, r).x, -1);
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
@@ -501,7 +510,7 @@ cudaError_t tc_setup(TcLaunch* out) {
 template <int MODE>
 cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const int4* segs,
                         int max_segs, int64_t dense_rows, const int32_t* crd, const float* vals, const float* X,
-                        const float* D, float* A, float* partial, cudaStream_t s) {
+                        const float* X2, const float* D, float* A, float* partial, cudaStream_t s) {
 #define SLNR_TC_CASE(KK, LL)                                                                              \
   if (K == KK && L == LL) {                                                                               \
     TcLaunch tl;                                                                                          \
@@ -511,8 +520,8 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
     if (grid > tl.grid_cap) grid = tl.grid_cap;                                                           \
     if (grid < 1) grid = 1;                                                                               \
     k_tc_gemm<KK, LL, MODE><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,              \
-                                                                         dense_rows, crd, vals, X, D, A,  \
-                                                                         partial);                        \
+                                                                         dense_rows, crd, vals, X, X2, D, \
+                                                                         A, partial);                     \
     return cudaGetLastError();                                                                            \
   }
   SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
@@ -546,16 +555,19 @@ cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t
 }
 
 cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, const float* D, float* A,
-                                const SegPlan& plan, cudaStream_t s) {
+                                const SegPlan& plan, cudaStream_t s, const float* C2) {
   if (B.nrows <= 0) return cudaSuccess;
+  if (C2 != nullptr)
+    return tc_dispatch<kSegmentsH>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, C,
+                                   C2, D, A, plan.partial, s);
   return tc_dispatch<kSegments>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                B.vals, C, D, A, plan.partial, s);
+                                B.vals, C, nullptr, D, A, plan.partial, s);
 }
 
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  return tc_dispatch<kDense>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, D, A, nullptr, s);
+  return tc_dispatch<kDense>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, D, A, nullptr, s);
 }
 
 }  // namespace slnr

@@ -32,11 +32,14 @@ def rel_err(gpu, ref, ref_abs) -> float:
     return float(np.max(diff[~zero] / ref_abs[~zero]))
 
 
+CSR_OPS = ("spmm_gemm", "sddmm_spmm", "sddmm_spmm_gemm", "spmmh_gemm")
+
+
 def to_device(w, device="cuda"):
     import torch
 
     import paper_2205_11622_gb300 as slnr
-    if w.op in ("spmm_gemm", "sddmm_spmm"):
+    if w.op in CSR_OPS:
         B = slnr.DeviceCSR.from_host(w.B, device)
     else:
         B = slnr.DeviceCSF3.from_host(w.B, device)
@@ -45,9 +48,9 @@ def to_device(w, device="cuda"):
 
 
 def output_rows(w) -> int:
-    if w.op in ("spmm_gemm", "sddmm_spmm"):
+    if w.op in CSR_OPS:
         return w.B.nrows
-    if w.op == "mttkrp":
+    if w.op in ("mttkrp", "mttkrp_gemm"):
         return w.B.dims[0]
     return w.B.nfibers
 
@@ -56,9 +59,15 @@ def values_of(op, out):
     return out[4] if op == "spttm_ttm" else out
 
 
-def uses_tensor_cores(op) -> bool:
-    return op in ("spmm_gemm", "spttm_ttm")
+def uses_tensor_cores(op, variant="fused") -> bool:
+    """Whether the call may contract on TF32 tensor cores when allowed: the
+    fused and unfused <SpMM,GEMM>, <SpTTM,SpTTM> and <SpMMH,GEMM>, and the
+    dense GEMM of the unfused <SDDMM,SpMM,GEMM> and <MTTKRP,GEMM> (their fused
+    consumers run in fp32)."""
+    if op in ("spmm_gemm", "spttm_ttm", "spmmh_gemm"):
+        return True
+    return variant == "unfused" and op in ("sddmm_spmm_gemm", "mttkrp_gemm")
 
 
-def tolerance(op, allow_tf32) -> float:
-    return TOL_TF32 if (allow_tf32 and uses_tensor_cores(op)) else TOL_FP32
+def tolerance(op, allow_tf32, variant="fused") -> float:
+    return TOL_TF32 if (allow_tf32 and uses_tensor_cores(op, variant)) else TOL_FP32

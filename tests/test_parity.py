@@ -40,7 +40,7 @@ def check(slnr, orc, w, variant="fused", allow_tf32=False, tol=None):
     ref, ref_abs = orc.run(w)
     got = P.values_of(w.op, out).cpu().numpy()
     err = P.rel_err(got, ref, ref_abs)
-    tol = tol if tol is not None else P.tolerance(w.op, allow_tf32)
+    tol = tol if tol is not None else P.tolerance(w.op, allow_tf32, variant)
     assert err <= tol, f"{w.name} {variant} tf32={allow_tf32}: err {err:.3e} > {tol:.1e}"
     if w.op == "spttm_ttm":
         p1, c1, p2, c2 = orc.spttm_ttm_pattern(w.B.crd1, w.B.pos2, w.B.crd2)

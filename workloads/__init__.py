@@ -213,7 +213,7 @@ def zipf_exponent_for_mean(max_len: int, mean_len: float) -> float:
 @dataclass
 class Workload:
     name: str
-    op: str                       # spmm_gemm | sddmm_spmm | mttkrp | spttm_ttm
+    op: str                       # spmm_gemm | sddmm_spmm | mttkrp | spttm_ttm | one of NEXT_OPS
     B: object                     # CSR or CSF3
     dense: dict = field(default_factory=dict)   # operand name -> fp32 array
     dims: dict = field(default_factory=dict)    # K, L, M as used by the op
@@ -285,6 +285,48 @@ def spttm_ttm_powerlaw(seed: int, dims, nnz: int, mean_len: float, max_len: int,
                     f"seed {seed:#x}")
 
 
+def sddmm_spmm_gemm_rmat(seed: int, n: int, deg: int, K: int, L: int, M: int, name="sddmm_spmm_gemm_rmat"):
+    """<SDDMM,SpMM,GEMM> A(i,m) = sum B(i,j) C(i,k) D(j,k) F(j,l) W(l,m); R-MAT, vals 1.0; C, D, F, W N(0,1)."""
+    r = Rng(seed)
+    pos, crd = rmat_csr_structure(r, n, n * deg)
+    vals = const(crd.shape[0], 1.0)
+    C = normal(r, (n, K))
+    D = normal(r, (n, K))
+    F = normal(r, (n, L))
+    W = normal(r, (L, M))
+    return Workload(name, "sddmm_spmm_gemm", CSR(n, n, pos, crd, vals), {"C": C, "D": D, "F": F, "W": W},
+                    {"K": K, "L": L, "M": M},
+                    f"B {n}x{n} R-MAT(.57,.19,.19,.05), {n * deg} distinct edges, vals 1.0; "
+                    f"C,D {n}x{K}, F {n}x{L}, W {L}x{M} N(0,1); seed {seed:#x}")
+
+
+def mttkrp_gemm_zipf(seed: int, dims, nnz: int, s: float, L: int, M: int, name="mttkrp_gemm_zipf"):
+    """<MTTKRP,GEMM> A(i,m) = sum B(i,j,k) C(j,l) D(k,l) E(l,m); Zipf(s) slices; vals U[0,1]; C, D, E U[-1,1]."""
+    r = Rng(seed)
+    bufs, ns, nfib = zipf_slices_csf_structure(r, dims, nnz, s)
+    vals = uniform(r, nnz, 0.0, 1.0)
+    B = _csf_from_buffers(dims, bufs, ns, nfib, nnz, vals)
+    C = uniform(r, (dims[1], L), -1.0, 1.0)
+    D = uniform(r, (dims[2], L), -1.0, 1.0)
+    E = uniform(r, (L, M), -1.0, 1.0)
+    return Workload(name, "mttkrp_gemm", B, {"C": C, "D": D, "E": E}, {"L": L, "M": M},
+                    f"B {dims[0]}x{dims[1]}x{dims[2]} CSF, {nnz} nnz, Zipf({s}) slice sizes, vals U[0,1]; "
+                    f"C {dims[1]}x{L}, D {dims[2]}x{L}, E {L}x{M} U[-1,1]; seed {seed:#x}")
+
+
+def spmmh_gemm_rmat(seed: int, n: int, deg: int, J: int, L: int, name="spmmh_gemm_rmat"):
+    """<SpMMH,GEMM> A(i,l) = sum B(i,k) C(k,j) D(k,j) E(j,l); R-MAT, vals U[-1,1]; C, D, E N(0,1)."""
+    r = Rng(seed)
+    pos, crd = rmat_csr_structure(r, n, n * deg)
+    vals = uniform(r, crd.shape[0], -1.0, 1.0)
+    C = normal(r, (n, J))
+    D = normal(r, (n, J))
+    E = normal(r, (J, L))
+    return Workload(name, "spmmh_gemm", CSR(n, n, pos, crd, vals), {"C": C, "D": D, "E": E}, {"J": J, "L": L},
+                    f"B {n}x{n} R-MAT(.57,.19,.19,.05), {n * deg} distinct edges, vals U[-1,1]; "
+                    f"C,D {n}x{J}, E {J}x{L} N(0,1); seed {seed:#x}")
+
+
 # The five benchmark workloads at full size (index = position in the benchmark
 # list).  `scale` < 1 shrinks the row count (R-MAT) or the nonzero count (CSF)
 # with the same recipe, for profiling captures on smaller cases.
@@ -320,4 +362,35 @@ def small(index: int, seed_offset: int = 100) -> Workload:
         return mttkrp_zipf(seed, (300, 200, 400), 60_000, 1.2, 32, name="mttkrp_zipf300")
     if index == 4:
         return spttm_ttm_powerlaw(seed, (150, 170, 400), 40_000, 8.0, 400, 64, 64, name="spttm_ttm_powerlaw400")
+    raise IndexError(index)
+
+
+# The further expressions of Sec. 6.2 (<SDDMM,SpMM,GEMM> with k,l,m = 64,64,64;
+# <MTTKRP,GEMM> with rank 32 and m = 64; <SpMMH,GEMM> with j,l = 128,128), on
+# the structures of the benchmark workloads above: index 0, 1, 2.
+NEXT_OPS = ("sddmm_spmm_gemm", "mttkrp_gemm", "spmmh_gemm")
+
+
+def next_full(index: int, scale: float = 1.0) -> Workload:
+    seed = SEED_BASE + 5 + index
+    tag = "" if scale == 1.0 else f"_x{scale:g}"
+    if index == 0:
+        return sddmm_spmm_gemm_rmat(seed, int(100_000 * scale), 20, 64, 64, 64,
+                                    name="sddmm_spmm_gemm_rmat100k_d20_64" + tag)
+    if index == 1:
+        return mttkrp_gemm_zipf(seed, (10_000, 10_000, 10_000), int(10_000_000 * scale), 1.2, 32, 64,
+                                name="mttkrp_gemm_zipf10k_10m_32_64" + tag)
+    if index == 2:
+        return spmmh_gemm_rmat(seed, int((1 << 20) * scale), 16, 128, 128, name="spmmh_gemm_rmat1m_d16_128" + tag)
+    raise IndexError(index)
+
+
+def next_small(index: int, seed_offset: int = 100) -> Workload:
+    seed = SEED_BASE + 5 + index + seed_offset
+    if index == 0:
+        return sddmm_spmm_gemm_rmat(seed, 3001, 20, 64, 64, 64, name="sddmm_spmm_gemm_rmat3001")
+    if index == 1:
+        return mttkrp_gemm_zipf(seed, (300, 200, 400), 60_000, 1.2, 32, 64, name="mttkrp_gemm_zipf300")
+    if index == 2:
+        return spmmh_gemm_rmat(seed, 5003, 16, 128, 128, name="spmmh_gemm_rmat5003")
     raise IndexError(index)
