@@ -15,6 +15,11 @@ GB/s (minimum bytes / time) are reported beside it.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl slnr|reference]
 
+--suite next times the three further expressions of Sec. 6.2 instead
+(<SDDMM,SpMM,GEMM> on the <SDDMM,SpMM> graph with k,l,m = 64; <MTTKRP,GEMM>
+on the MTTKRP tensor with rank 32 and m = 64; <SpMMH,GEMM> on the 2^20 R-MAT
+graph with j,l = 128), with the same JSON line.
+
 Under torchrun each rank runs an independent replica on its own GPU (the
 expressions need no exchange between GPUs); value = all ranks' flops / the
 slowest rank's time.  --impl reference times the CPU oracle instead (on rank 0).
@@ -40,6 +45,7 @@ if ROOT not in sys.path:
 import workloads as wl  # noqa: E402
 
 BENCH_CONFIGS = (1, 2, 3, 4)   # full-size workloads timed in one step (index 0 is the small parity case)
+CSR_OPS = ("spmm_gemm", "sddmm_spmm", "sddmm_spmm_gemm", "spmmh_gemm")
 
 
 # ---------------------------------------------------------------------------
@@ -53,7 +59,7 @@ def _distinct(a) -> int:
 
 def row_sizes(w):
     """Work units of each expression's output rows and their nonzero counts."""
-    if w.op in ("spmm_gemm", "sddmm_spmm"):
+    if w.op in CSR_OPS:
         return np.diff(w.B.pos).astype(np.int64)
     if w.op == "spttm_ttm":
         return np.diff(w.B.pos3).astype(np.int64)
@@ -73,7 +79,7 @@ def row_flops(w) -> np.ndarray:
     if w.op == "sddmm_spmm":     # per nonzero: dot (2L), scale (1), axpy (2K)
         n = np.diff(w.B.pos).astype(np.int64)
         return n * (2 * d["L"] + 1 + 2 * d["K"])
-    if w.op == "mttkrp":         # 2 nnz L + 2 nfibers L, per slice
+    if w.op in ("mttkrp", "mttkrp_gemm"):  # 2 nnz L + 2 nfibers L per slice (+ 2 L M per slice)
         L = d["L"]
         f = np.zeros(w.B.dims[0], np.int64)
         if w.B.nslices:
@@ -81,7 +87,15 @@ def row_flops(w) -> np.ndarray:
             nnz_s = np.add.reduceat(fib_nnz, w.B.pos2[:-1]) if w.B.nfibers else np.zeros(w.B.nslices, np.int64)
             nfib_s = np.diff(w.B.pos2).astype(np.int64)
             f[w.B.crd1] = 2 * nnz_s * L + 2 * nfib_s * L
+            if w.op == "mttkrp_gemm":
+                f[w.B.crd1] += 2 * L * d["M"]
         return f
+    if w.op == "sddmm_spmm_gemm":  # per nonzero: dot (2K), scale (1), axpy (2L); 2 L M per non-empty row
+        n = np.diff(w.B.pos).astype(np.int64)
+        return n * (2 * d["K"] + 1 + 2 * d["L"]) + 2 * (n > 0) * d["L"] * d["M"]
+    if w.op == "spmmh_gemm":     # per nonzero: Hadamard product and axpy (3J); 2 J L per non-empty row
+        n = np.diff(w.B.pos).astype(np.int64)
+        return 3 * n * d["J"] + 2 * (n > 0) * d["J"] * d["L"]
     if w.op == "spttm_ttm":      # 2 nnz L + 2 L M per fiber
         n = np.diff(w.B.pos3).astype(np.int64)
         return 2 * n * d["L"] + 2 * d["L"] * d["M"]
@@ -104,7 +118,18 @@ def min_bytes(w) -> int:
         nonempty = int(np.count_nonzero(np.diff(B.pos)))
         cols = _distinct(B.crd)
         return 4 * (B.nrows + 1) + 8 * B.nnz + 4 * L * nonempty + 4 * (L + K) * cols + 4 * B.nrows * K
+    if w.op == "sddmm_spmm_gemm":
+        K, L, M = d["K"], d["L"], d["M"]
+        nonempty = int(np.count_nonzero(np.diff(B.pos)))
+        cols = _distinct(B.crd)
+        return 4 * (B.nrows + 1) + 8 * B.nnz + 4 * K * nonempty + 4 * (K + L) * cols + 4 * L * M + 4 * B.nrows * M
+    if w.op == "spmmh_gemm":
+        J, L = d["J"], d["L"]
+        return 4 * (B.nrows + 1) + 8 * B.nnz + 8 * J * _distinct(B.crd) + 4 * J * L + 4 * B.nrows * L
     structure = 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers + 4 * (B.nfibers + 1) + 8 * B.nnz
+    if w.op == "mttkrp_gemm":
+        L, M = d["L"], d["M"]
+        return structure + 4 * L * (_distinct(B.crd2) + _distinct(B.crd3)) + 4 * L * M + 4 * B.dims[0] * M
     if w.op == "mttkrp":
         L = d["L"]
         return structure + 4 * L * (_distinct(B.crd2) + _distinct(B.crd3)) + 4 * B.dims[0] * L
@@ -265,7 +290,7 @@ def run_reference(args, rank, world):
     secs = sum(times)
     value = flops_total / secs / 1e9
     line = {
-        "impl": "reference", "metric": "useful GFLOP/s (4 fused sparse expressions)", "value": round(value, 4),
+        "impl": "reference", "metric": metric_name(args), "value": round(value, 4),
         "unit": "GFLOP/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(1e3 * secs / args.steps, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -281,11 +306,20 @@ def run_reference(args, rank, world):
 
 
 def select_workloads(args):
-    ws = [wl.full(i, args.scale) for i in BENCH_CONFIGS]
+    if args.suite == "next":
+        ws = [wl.next_full(i, args.scale) for i in range(len(wl.NEXT_OPS))]
+    else:
+        ws = [wl.full(i, args.scale) for i in BENCH_CONFIGS]
     ws = [w for w in ws if args.expr in w.name]
     if not ws:
         raise SystemExit(f"no workload matches --expr {args.expr!r}")
     return ws
+
+
+def metric_name(args):
+    if args.suite == "next":
+        return "useful GFLOP/s (3 further fused sparse expressions of Sec. 6.2)"
+    return "useful GFLOP/s (4 fused sparse expressions)"
 
 
 def config_block(ws):
@@ -312,6 +346,9 @@ def main():
     ap.add_argument("--ref-gflop-per-expr", type=float, default=1.0)
     ap.add_argument("--expr", default="", help="only the expressions whose name contains this (profiling)")
     ap.add_argument("--scale", type=float, default=1.0, help="shrink the workloads (profiling captures)")
+    ap.add_argument("--suite", choices=["main", "next"], default="main",
+                    help="main: the four benchmark expressions (the step); next: <SDDMM,SpMM,GEMM>, "
+                         "<MTTKRP,GEMM>, <SpMMH,GEMM> at full size")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -340,7 +377,7 @@ def main():
 
     # device-resident inputs, preallocated outputs and workspaces
     def upload(w):
-        if w.op in ("spmm_gemm", "sddmm_spmm"):
+        if w.op in CSR_OPS:
             B = slnr.DeviceCSR.from_host(w.B, dev)
         else:
             B = slnr.DeviceCSF3.from_host(w.B, dev)
@@ -442,7 +479,7 @@ def main():
         e2e = measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, args.steps, total_flops, world, pg, dev)
 
     line = {
-        "metric": "useful GFLOP/s (4 fused sparse expressions)", "value": round(value, 2), "unit": "GFLOP/s",
+        "metric": metric_name(args), "value": round(value, 2), "unit": "GFLOP/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32 (tf32 tensor-core contractions allowed)" if allow_tf32 else "f32",
@@ -464,7 +501,7 @@ def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_fl
     host_in, dev_in, host_out, dev_out = [], [], [], []
     for i, w in enumerate(ws):
         B, dense = dev_inputs[i]
-        arrays = [getattr(B, f) for f in ("pos", "crd", "vals")] if w.op in ("spmm_gemm", "sddmm_spmm") else \
+        arrays = [getattr(B, f) for f in ("pos", "crd", "vals")] if w.op in CSR_OPS else \
             [getattr(B, f) for f in ("pos1", "crd1", "pos2", "crd2", "pos3", "crd3", "vals")]
         arrays += list(dense.values())
         for a in arrays:
