@@ -83,12 +83,12 @@ struct RowLanes {
 
 template <int VPL>
 __device__ __forceinline__ void ldg_vec(float (&v)[VPL], const float* __restrict__ p) {
+  static_assert(VPL % 4 == 0, "whole float4s");
   const float4* q = reinterpret_cast<const float4*>(p);
-  float4 a = __ldg(q);
-  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-  if constexpr (VPL == 8) {
-    float4 b = __ldg(q + 1);
-    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+#pragma unroll
+  for (int h = 0; h < VPL / 4; ++h) {
+    const float4 a = __ldg(q + h);
+    v[4 * h] = a.x; v[4 * h + 1] = a.y; v[4 * h + 2] = a.z; v[4 * h + 3] = a.w;
   }
 }
 

@@ -194,7 +194,7 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 }
 
 #ifndef SLNR_TC_VPL
-#define SLNR_TC_VPL 4  // T-row columns per producer lane (4 or 8)
+#define SLNR_TC_VPL 4  // T-row columns per producer lane (4, 8 or 16)
 #endif
 #ifndef SLNR_TC_UNROLL
 #define SLNR_TC_UNROLL 8  // gathered rows in flight per lane group
@@ -208,13 +208,94 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 // float4s; a warp builds G = 32 / GS rows at once, one per group, with U row
 // gathers in flight per group.  A claim is the G consecutive items of one
 // warp pass.
+#ifndef SLNR_TC_PF_AHEAD
+#define SLNR_TC_PF_AHEAD 8  // rows of a segment prefetched into L2 beyond the batch in flight
+#endif
+
+// L2 prefetch of the 128-byte line holding p (no register, nothing to wait for).
+__device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+
+// acc += sum_{p in [p0,p1)} vals[p] * R(crd[p])[col .. col+VPL), sequential in p,
+// where R(k) = X[k,:] (or X[k,:] .* X2[k,:] with H).  U rows are loaded per
+// batch (the last batch predicated, so a short segment costs one round trip
+// per batch, not per row).  Rows further ahead are pulled into L2 by line
+// prefetches, which hold no register: each of the group's GS lanes prefetches
+// one 128-byte line, RPI = GS / LPR rows per step, and the front is kept AHEAD
+// rows beyond the batch in flight.
+template <int K, int VPL, int U, int AHEAD, bool H>
+__device__ __forceinline__ void gather_pf(float (&acc)[VPL], const int32_t* __restrict__ crd,
+                                          const float* __restrict__ vals, int p0, int p1,
+                                          const float* __restrict__ X, const float* __restrict__ X2, int col,
+                                          int gl) {
+  constexpr int GS = K / VPL, LPR = K / 32, RPI = GS / LPR;
+  static_assert(AHEAD % RPI == 0, "the prefetch window is whole steps");
+  constexpr int NPF = AHEAD / RPI;
+  const int prow = gl / LPR, poff = (gl % LPR) * 32;
+  auto pf_row = [&](int c) {
+    prefetch_line(X + (int64_t)c * K + poff);
+    if constexpr (H) prefetch_line(X2 + (int64_t)c * K + poff);
+  };
+  int pq = p0 + U;  // first row not covered by the first batch or the window
+  int pf = -1;      // coordinate of row pq + prow (the next prefetch step)
+  if constexpr (NPF > 0) {
+    int cs[NPF];
+#pragma unroll
+    for (int k = 0; k < NPF; ++k) {
+      const int q = pq + k * RPI + prow;
+      cs[k] = q < p1 ? __ldg(crd + q) : -1;
+    }
+    pq += AHEAD;
+    pf = pq + prow < p1 ? __ldg(crd + pq + prow) : -1;
+#pragma unroll
+    for (int k = 0; k < NPF; ++k)
+      if (cs[k] >= 0) pf_row(cs[k]);
+  }
+  for (int p = p0; p < p1; p += U) {
+    if constexpr (NPF > 0) {
+      if (pq < p + U + AHEAD && pq < p1) {  // advance the front by one step
+        if (pf >= 0) pf_row(pf);
+        pq += RPI;
+        pf = pq + prow < p1 ? __ldg(crd + pq + prow) : -1;
+      }
+    }
+    int c[U];
+    float v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const bool ok = p + u < p1;
+      c[u] = ok ? __ldg(crd + p + u) : -1;
+      v[u] = ok ? __ldg(vals + p + u) : 0.f;
+    }
+    float x[U][VPL];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (c[u] >= 0) {
+        ldg_vec<VPL>(x[u], X + (int64_t)c[u] * K + col);
+        if constexpr (H) {
+          float x2[VPL];
+          ldg_vec<VPL>(x2, X2 + (int64_t)c[u] * K + col);
+#pragma unroll
+          for (int e = 0; e < VPL; ++e) x[u][e] *= x2[e];
+        }
+      } else {
+        zero_vec(x[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (c[u] >= 0)
+#pragma unroll
+        for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v[u], x[u][e], acc[e]);
+  }
+}
+
 template <int K>
 struct ProdLayout {
   static constexpr int VPL = K / SLNR_TC_VPL >= 1 && K / SLNR_TC_VPL <= 32 ? SLNR_TC_VPL : 4;
   static constexpr int GS = K / VPL;
   static constexpr int G = 32 / GS;
   static constexpr int U = SLNR_TC_UNROLL;
-  static_assert(VPL == 4 || VPL == 8, "VPL must be 4 or 8");
+  static_assert(VPL == 4 || VPL == 8 || VPL == 16, "VPL must be 4, 8 or 16");
   static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
 };
 
@@ -248,10 +329,17 @@ __device__ __forceinline__ void store_t_part(uint8_t* sTb, int s, int col, const
 // completed tiles that the epilogue publishes (release) once all four
 // epilogue warps have read the tile's row destinations.  Every wait is
 // bounded; a timeout raises kErrTimeout and the CTA winds down.
+// Items per producer claim: one per lane group (a segment), or
+// SLNR_TC_DENSE_ROWS per lane group in DENSE mode.
+template <int K, int MODE>
+__host__ __device__ constexpr int claim_items() {
+  return ProdLayout<K>::G * (MODE == kDense ? SLNR_TC_DENSE_ROWS : 1);
+}
+
 constexpr int kProducerWarps = 27;
 constexpr int kMmaWarp = 27;  // warps 28..31: epilogue
 
-template <int K, int L, int MODE>
+template <int K, int L, int MODE, bool PF>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_gemm(WsHeader* hdr, const int4* __restrict__ segs, int max_segs,
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
@@ -282,7 +370,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   if (tid == 0) {
     for (int b = 0; b < NBUF; ++b) {
-      tc::mbar_init(&full_bar[b], kTcRows / (PL::G * (MODE != kDense ? 1 : SLNR_TC_DENSE_ROWS)));  // one arrival per claim
+      tc::mbar_init(&full_bar[b], kTcRows / claim_items<K, MODE>());  // one arrival per claim
       tc::mbar_init(&mma_bar[b], 1);
       tc::mbar_init(&free_bar[b], 4);
       last_commit[b] = -1;
@@ -329,6 +417,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // destinations, and lane 0 arrives once for the claim.
     constexpr int VPL = PL::VPL, G = PL::G, R = MODE != kDense ? 1 : SLNR_TC_DENSE_ROWS;
     constexpr int IPC = G * R, CPT = kTcRows / IPC;
+    static_assert(IPC == claim_items<K, MODE>(), "barrier count matches the claims");
     static_assert(kTcRows % IPC == 0, "claims tile the item tile");
     const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
     const int nclaims = nlocal * CPT;
@@ -354,11 +443,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if constexpr (MODE != kDense) {
         const int4 rec_next = load_rec(cl_next, 0);  // loads while this claim is built
         zero_vec(acc[0]);
+        constexpr bool H = MODE == kSegmentsH;
+        constexpr int UG = H ? PL::U / 2 : PL::U;  // two loads per nonzero in Hadamard mode
         if (rec.x >= 0) {
-          if constexpr (MODE == kSegmentsH)
-            gather_acc<VPL, PL::U / 2, true>(acc[0], crd, vals, rec.y, rec.z, X, K, col, X2);
+          if constexpr (PF)
+            gather_pf<K, VPL, UG, SLNR_TC_PF_AHEAD, H>(acc[0], crd, vals, rec.y, rec.z, X, X2, col, lane % PL::GS);
           else
-            gather_acc<VPL, PL::U>(acc[0], crd, vals, rec.y, rec.z, X, K, col);
+            gather_acc<VPL, UG, H>(acc[0], crd, vals, rec.y, rec.z, X, K, col, X2);
         }
         dst0 = make_int2(rec.x, rec.w);
         rec = rec_next;
@@ -470,7 +561,7 @@ struct TcLaunch {
   size_t smem;
 };
 
-template <int K, int L, int MODE>
+template <int K, int L, int MODE, bool PF>
 cudaError_t tc_setup(TcLaunch* out) {
   static TcLaunch cached[64] = {};
   int dev = 0;
@@ -489,14 +580,14 @@ cudaError_t tc_setup(TcLaunch* out) {
   const int max_ctas = 512 / (tc_nbuf(K, L) * L);
   const size_t floor_bytes = (size_t)sm_smem / (size_t)(max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
-  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
+  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE, PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
       cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE, PF>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                 (int)cudaSharedmemCarveoutMaxShared)) != cudaSuccess)
     return e;
   int occ = 0;
-  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_tc_gemm<K, L, MODE>, kTcThreads, smem)) !=
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_tc_gemm<K, L, MODE, PF>, kTcThreads, smem)) !=
       cudaSuccess)
     return e;
   if (occ < 1) return cudaErrorInvalidConfiguration;
@@ -507,21 +598,21 @@ cudaError_t tc_setup(TcLaunch* out) {
   return cudaSuccess;
 }
 
-template <int MODE>
+template <int MODE, bool PF>
 cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const int4* segs,
                         int max_segs, int64_t dense_rows, const int32_t* crd, const float* vals, const float* X,
                         const float* X2, const float* D, float* A, float* partial, cudaStream_t s) {
 #define SLNR_TC_CASE(KK, LL)                                                                              \
   if (K == KK && L == LL) {                                                                               \
     TcLaunch tl;                                                                                          \
-    cudaError_t e = tc_setup<KK, LL, MODE>(&tl);                                                          \
+    cudaError_t e = tc_setup<KK, LL, MODE, PF>(&tl);                                                      \
     if (e != cudaSuccess) return e;                                                                       \
     int64_t grid = (items_upper + kTcRows - 1) / kTcRows;                                                 \
     if (grid > tl.grid_cap) grid = tl.grid_cap;                                                           \
     if (grid < 1) grid = 1;                                                                               \
-    k_tc_gemm<KK, LL, MODE><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,              \
-                                                                         dense_rows, crd, vals, X, X2, D, \
-                                                                         A, partial);                     \
+    k_tc_gemm<KK, LL, MODE, PF><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,          \
+                                                                             dense_rows, crd, vals, X,    \
+                                                                             X2, D, A, partial);          \
     return cudaGetLastError();                                                                            \
   }
   SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
@@ -529,6 +620,19 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
   SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128)
 #undef SLNR_TC_CASE
   return cudaErrorInvalidValue;
+}
+
+// L2 size of the current device (cached per device; 0 if it cannot be read).
+size_t l2_bytes() {
+  static size_t cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev) != cudaSuccess) return 0;
+    cached[dev] = (size_t)v;
+  }
+  return cached[dev];
 }
 
 }  // namespace
@@ -557,17 +661,24 @@ cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t
 cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, const float* D, float* A,
                                 const SegPlan& plan, cudaStream_t s, const float* C2) {
   if (B.nrows <= 0) return cudaSuccess;
+  // Gathered rows that do not fit in half of L2 miss often: the producers
+  // then prefetch the rows ahead of their gathers into L2 (gather_pf).
+  const bool pf = (size_t)B.ncols * (size_t)K * sizeof(float) * (C2 != nullptr ? 2 : 1) > l2_bytes() / 2;
   if (C2 != nullptr)
-    return tc_dispatch<kSegmentsH>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, C,
-                                   C2, D, A, plan.partial, s);
-  return tc_dispatch<kSegments>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                B.vals, C, nullptr, D, A, plan.partial, s);
+    return pf ? tc_dispatch<kSegmentsH, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
+                                              B.vals, C, C2, D, A, plan.partial, s)
+              : tc_dispatch<kSegmentsH, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
+                                               B.vals, C, C2, D, A, plan.partial, s);
+  return pf ? tc_dispatch<kSegments, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
+                                           B.vals, C, nullptr, D, A, plan.partial, s)
+            : tc_dispatch<kSegments, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
+                                            B.vals, C, nullptr, D, A, plan.partial, s);
 }
 
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  return tc_dispatch<kDense>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, D, A, nullptr, s);
+  return tc_dispatch<kDense, false>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, D, A, nullptr, s);
 }
 
 }  // namespace slnr

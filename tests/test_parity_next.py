@@ -156,3 +156,14 @@ def test_fused_is_deterministic_and_agrees_with_unfused(slnr, orc):
         assert torch.equal(a, b), f"{w.name}: two fused runs differ"
         _, ref_abs = orc.run(w)
         assert P.rel_err(c.cpu().numpy(), a.cpu().numpy().astype(np.float64), ref_abs) <= 2 * P.TOL_FP32
+
+
+def test_spmmh_gemm_gathered_matrices_larger_than_l2(slnr, orc):
+    # C and D have 2^20 rows of 128 floats: the Hadamard producers prefetch ahead
+    r = wl.Rng(0x51A4 + 77)
+    n, ncols, J, L = 2001, 1 << 20, 128, 64
+    pos, crd = wl.uniform_csr_structure(r, n, ncols, 19)
+    vals = wl.uniform(r, crd.shape[0], -1.0, 1.0)
+    dense = {"C": wl.normal(r, (ncols, J)), "D": wl.normal(r, (ncols, J)), "E": wl.normal(r, (J, L))}
+    w = wl.Workload("spmmh_gemm_wide", "spmmh_gemm", wl.CSR(n, ncols, pos, crd, vals), dense, {"J": J, "L": L})
+    check(slnr, orc, w, "fused", True)
