@@ -31,7 +31,8 @@ struct WsHeader {        // first 256 bytes of every workspace
   int n_units;           // MTTKRP units
   int error;             // validation / runtime flags (bit set = problem found)
   int n_segs;            // segments of the tensor-core path
-  int pad[59];
+  int next_tile;         // tensor-core path: next item tile to hand to a CTA
+  int pad[58];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 

@@ -170,11 +170,32 @@ __device__ __forceinline__ bool count_wait_timeout(const int* count, int target)
   return true;
 }
 
+#ifndef SLNR_TC_MBAR_SLEEP
+#define SLNR_TC_MBAR_SLEEP 256  // back-off (ns) between polls of an mbarrier by the MMA and epilogue warps
+#endif
+
+// Waits for the phase with the given parity to complete; false on timeout.
+// Sleeps between polls so that the waiting MMA and epilogue warps leave the
+// issue slots to the producers (their work has slack of a whole tile).
 __device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity) {
   const long long t0 = clock64();
-  while (!tc::mbar_try_wait(bar, parity))
+  while (!tc::mbar_try_wait(bar, parity)) {
+    if (SLNR_TC_MBAR_SLEEP > 0) __nanosleep(SLNR_TC_MBAR_SLEEP);
     if (clock64() - t0 > kWaitCycles) return false;
+  }
   return true;
+}
+
+// Waits for the phase with the given parity to complete (1), or until
+// *end <= j, i.e. there is no tile j to wait for (0); -1 on timeout.
+__device__ __forceinline__ int mbar_wait_or_end(uint64_t* bar, uint32_t parity, const int* end, int j) {
+  const long long t0 = clock64();
+  while (!tc::mbar_try_wait(bar, parity)) {
+    if (*reinterpret_cast<const volatile int*>(end) <= j) return 0;
+    if (SLNR_TC_MBAR_SLEEP > 0) __nanosleep(SLNR_TC_MBAR_SLEEP);
+    if (clock64() - t0 > kWaitCycles) return -1;
+  }
+  return 1;
 }
 
 // kSegments: gathered row segments; kSegmentsH: the same with Hadamard rows
@@ -337,6 +358,7 @@ __host__ __device__ constexpr int claim_items() {
 }
 
 constexpr int kProducerWarps = 27;
+constexpr int kTileRing = 16;  // local tiles whose global index is kept in shared memory
 constexpr int kMmaWarp = 27;  // warps 28..31: epilogue
 
 template <int K, int L, int MODE, bool PF>
@@ -358,7 +380,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ uint64_t full_bar[NBUF], mma_bar[NBUF], free_bar[NBUF];
   __shared__ int2 dest[NBUF][kTcRows];  // per slot: (A row, partial slot); x < 0 = padding
   __shared__ uint32_t tmem_base;
-  __shared__ int claim, fail_flag, mma_tiles_done;
+  __shared__ int claim, fill, fail_flag, mma_tiles_done;
+  __shared__ int tile_gid[kTileRing], tile_seq[kTileRing], end_tile;
   __shared__ int last_commit[NBUF];     // last tile committed to each accumulator (-1: none)
   uint8_t* sT = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sD = sT + NBUF * TBYTES;
@@ -377,8 +400,31 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     tc::fence_mbar_init();
     claim = 0;
+    fill = 0;
     fail_flag = 0;
     mma_tiles_done = 0;
+  }
+  // Item tiles are handed out dynamically: CTAs take them from a global
+  // counter in the workspace header (zeroed before the launch), one tile
+  // ahead of need, so the hub rows' costly tiles do not pile up on a few SMs.
+  // Local tile j's global index is published in a small shared ring
+  // (tile_gid, with tile_seq = j + 1 once written); the first local tile
+  // whose index lies past the last item tile is end_tile, and every role
+  // stops there.
+  int64_t nitems;
+  if (MODE != kDense) {
+    const int n = hdr->n_segs;
+    nitems = n < max_segs ? n : max_segs;
+  } else {
+    nitems = dense_rows;
+  }
+  const int64_t ntiles = (nitems + kTcRows - 1) / kTcRows;
+  if (tid == 0) {
+    for (int r = 0; r < kTileRing; ++r) tile_seq[r] = 0;
+    const int g0 = atomicAdd(&hdr->next_tile, 1);
+    tile_gid[0] = g0;
+    tile_seq[0] = 1;
+    end_tile = g0 >= ntiles ? 0 : INT_MAX;
   }
   // D (K x L, row-major) -> D^T as the B operand (L rows of K), tf32
   for (int i = tid; i < K * (L / 4); i += kTcThreads) {
@@ -395,16 +441,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   tc::tc_fence_after_sync();
   const uint32_t tmem = tmem_base;
 
-  int64_t nitems;
-  if (MODE != kDense) {
-    const int n = hdr->n_segs;
-    nitems = n < max_segs ? n : max_segs;
-  } else {
-    nitems = dense_rows;
-  }
-  const int64_t ntiles = (nitems + kTcRows - 1) / kTcRows;
-  // this CTA's items: rows of item tiles blockIdx.x + j * gridDim.x, j < nlocal
-  const int nlocal = (int)(ntiles > blockIdx.x ? (ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0);
+  // global item tile of local tile t: >= 0 once known, -1 if t does not
+  // exist (t >= end_tile), -2 if the wait timed out
+  auto tile_of = [&](int t) -> int {
+    const long long t0 = clock64();
+    while (tc::ld_acquire_smem(&tile_seq[t % kTileRing]) != t + 1) {
+      if (*reinterpret_cast<volatile int*>(&end_tile) <= t) return -1;
+      __nanosleep(32);
+      if (clock64() - t0 > kWaitCycles) return -2;
+    }
+    const int gid = *reinterpret_cast<volatile int*>(&tile_gid[t % kTileRing]);
+    return gid < ntiles ? gid : -1;
+  };
+  // the first claim of local tile t fetches the global index of tile t + 1
+  auto fetch_next_tile = [&](int t) {
+    const int gnext = atomicAdd(&hdr->next_tile, 1);
+    tile_gid[(t + 1) % kTileRing] = gnext;
+    if (gnext >= ntiles) atomicMin(&end_tile, t + 1);
+    tc::st_release_smem(&tile_seq[(t + 1) % kTileRing], t + 2);
+  };
 
   if (warp < kProducerWarps) {
     // ---------------- producers ----------------
@@ -420,28 +475,43 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     static_assert(IPC == claim_items<K, MODE>(), "barrier count matches the claims");
     static_assert(kTcRows % IPC == 0, "claims tile the item tile");
     const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
-    const int nclaims = nlocal * CPT;
-    auto load_rec = [&](int c, int r) -> int4 {
+    // record of item g + r G of claim c, whose item tile has global index gid
+    auto load_rec = [&](int gid, int c, int r) -> int4 {
       int4 rv = make_int4(-1, 0, 0, -1);
-      if (c < nclaims) {
-        const int64_t item =
-            ((int64_t)blockIdx.x + (int64_t)(c / CPT) * gridDim.x) * kTcRows + (c % CPT) * IPC + r * G + g;
-        if (item < nitems) rv = (MODE != kDense) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
-      }
+      const int64_t item = (int64_t)gid * kTcRows + (c % CPT) * IPC + r * G + g;
+      if (item < nitems) rv = (MODE != kDense) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
       return rv;
     };
-    int x = 0;
-    if (lane == 0) x = atomicAdd(&claim, 1);
-    int cl = __shfl_sync(0xffffffffu, x, 0);
-    int4 rec = load_rec(cl, 0);  // segment record (R = 1)
-    while (cl < nclaims) {
-      x = 0;
-      if (lane == 0) x = atomicAdd(&claim, 1);
-      const int cl_next = __shfl_sync(0xffffffffu, x, 0);
+    // takes the next claim of this CTA; returns its item tile's global index
+    // (< 0: no such tile / timeout).  The first claim of a local tile also
+    // fetches the next local tile's global index.
+    int known_tile = -1, known_gid = -1;  // the last local tile this warp resolved
+    auto take_claim = [&](int& c) -> int {
+      int v = 0;
+      if (lane == 0) v = atomicAdd(&claim, 1);
+      c = __shfl_sync(0xffffffffu, v, 0);
+      const int t = c / CPT;
+      if (t != known_tile) {
+        known_gid = __shfl_sync(0xffffffffu, tile_of(t), 0);
+        known_tile = known_gid >= 0 ? t : -1;
+      }
+      const int gid = known_gid;
+      if (gid >= 0 && c % CPT == 0) {
+        if (lane == 0) fetch_next_tile(t);
+        __syncwarp();
+      }
+      return gid;
+    };
+    int cl = 0;
+    int gid = take_claim(cl);
+    int4 rec = gid >= 0 ? load_rec(gid, cl, 0) : make_int4(-1, 0, 0, -1);  // segment record (R = 1)
+    while (gid >= 0) {
+      int cl_next = 0;
+      const int gid_next = take_claim(cl_next);
       float acc[R][VPL];
       int2 dst0 = make_int2(-1, -1);  // destination of the segment (R = 1)
       if constexpr (MODE != kDense) {
-        const int4 rec_next = load_rec(cl_next, 0);  // loads while this claim is built
+        const int4 rec_next = gid_next >= 0 ? load_rec(gid_next, cl_next, 0) : make_int4(-1, 0, 0, -1);
         zero_vec(acc[0]);
         constexpr bool H = MODE == kSegmentsH;
         constexpr int UG = H ? PL::U / 2 : PL::U;  // two loads per nonzero in Hadamard mode
@@ -456,12 +526,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       } else {
 #pragma unroll
         for (int r = 0; r < R; ++r) {
-          const int4 rr = load_rec(cl, r);
+          const int4 rr = load_rec(gid, cl, r);
           if (rr.x >= 0) ldg_vec<VPL>(acc[r], X + (int64_t)rr.x * K + col); else zero_vec(acc[r]);
         }
       }
       __syncwarp();
-      const int j = cl / CPT, b = j % NBUF, s0 = (cl % CPT) * IPC + g;
+      // the claim's IPC rows take the next IPC slots in completion order, so a
+      // long segment delays only its own rows, never a whole tile (the item
+      // tiles of this CTA, and the slot tiles the MMAs consume, are as many)
+      int sl = 0;
+      if (lane == 0) sl = atomicAdd(&fill, IPC);
+      sl = __shfl_sync(0xffffffffu, sl, 0);
+      const int j = sl / kTcRows, b = j % NBUF, s0 = sl % kTcRows + g;
       if (j >= NBUF) {
         const bool ok = count_wait_timeout(&mma_tiles_done, j - NBUF + 1);
         if (!__all_sync(0xffffffffu, ok)) {
@@ -473,21 +549,28 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int r = 0; r < R; ++r) {
         store_t_part<VPL>(sT + b * TBYTES, s0 + r * G, col, acc[r]);
         if (lane % PL::GS == 0)
-          dest[b][s0 + r * G] = MODE != kDense ? dst0 : make_int2(load_rec(cl, r).x, -1);
+          dest[b][s0 + r * G] = MODE != kDense ? dst0 : make_int2(load_rec(gid, cl, r).x, -1);
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&full_bar[b]);
+      if (gid_next == -2) {  // timed out waiting for a tile index
+        atomicOr(&fail_flag, 1);
+        break;
+      }
       cl = cl_next;
+      gid = gid_next;
     }
+    if (gid == -2) atomicOr(&fail_flag, 1);
   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t sT_addr = tc::smem_u32(sT), sD_addr = tc::smem_u32(sD);
-      for (int j = 0; j < nlocal; ++j) {
+      for (int j = 0;; ++j) {
         const int b = j % NBUF;
-        if (!mbar_wait_timeout(&full_bar[b], (j / NBUF) & 1) ||
-            (j >= NBUF && !mbar_wait_timeout(&free_bar[b], ((j / NBUF) - 1) & 1))) {
+        const int st = mbar_wait_or_end(&full_bar[b], (j / NBUF) & 1, &end_tile, j);
+        if (st == 0) break;  // this CTA has no tile j
+        if (st < 0 || (j >= NBUF && !mbar_wait_timeout(&free_bar[b], ((j / NBUF) - 1) & 1))) {
           atomicOr(&fail_flag, 1);
           break;
         }
@@ -509,10 +592,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else {
     // ---------------- epilogue ----------------
     const int q = warp & 3;  // TMEM lane quadrant of this warp
-    for (int j = 0; j < nlocal; ++j) {
+    for (int j = 0;; ++j) {
       const int b = j % NBUF;
-      const bool ok = mbar_wait_timeout(&mma_bar[b], (j / NBUF) & 1);
-      if (!__all_sync(0xffffffffu, ok)) {
+      const int st = __shfl_sync(0xffffffffu, mbar_wait_or_end(&mma_bar[b], (j / NBUF) & 1, &end_tile, j), 0);
+      if (st == 0) break;  // this CTA has no tile j
+      if (st < 0) {
         atomicOr(&fail_flag, 1);
         break;
       }
@@ -610,6 +694,7 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
     int64_t grid = (items_upper + kTcRows - 1) / kTcRows;                                                 \
     if (grid > tl.grid_cap) grid = tl.grid_cap;                                                           \
     if (grid < 1) grid = 1;                                                                               \
+    if ((e = cudaMemsetAsync(&hdr->next_tile, 0, sizeof(int), s)) != cudaSuccess) return e;               \
     k_tc_gemm<KK, LL, MODE, PF><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,          \
                                                                              dense_rows, crd, vals, X,    \
                                                                              X2, D, A, partial);          \
