@@ -229,6 +229,9 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 // float4s; a warp builds G = 32 / GS rows at once, one per group, with U row
 // gathers in flight per group.  A claim is the G consecutive items of one
 // warp pass.
+#ifndef SLNR_TC_TAIL_BATCH
+#define SLNR_TC_TAIL_BATCH 1  // segments without prefetch: the last batch loaded at once (0: row by row)
+#endif
 #ifndef SLNR_TC_PF_AHEAD
 #define SLNR_TC_PF_AHEAD 8  // rows of a segment prefetched into L2 beyond the batch in flight
 #endif
@@ -271,14 +274,45 @@ __device__ __forceinline__ void gather_pf(float (&acc)[VPL], const int32_t* __re
     for (int k = 0; k < NPF; ++k)
       if (cs[k] >= 0) pf_row(cs[k]);
   }
-  for (int p = p0; p < p1; p += U) {
+  // advances the prefetch front by one step when it is within AHEAD rows of p + U
+  auto advance = [&](int p) {
     if constexpr (NPF > 0) {
-      if (pq < p + U + AHEAD && pq < p1) {  // advance the front by one step
+      if (pq < p + U + AHEAD && pq < p1) {
         if (pf >= 0) pf_row(pf);
         pq += RPI;
         pf = pq + prow < p1 ? __ldg(crd + pq + prow) : -1;
       }
     }
+  };
+  auto row = [&](float (&x)[VPL], int c) {
+    ldg_vec<VPL>(x, X + (int64_t)c * K + col);
+    if constexpr (H) {
+      float x2[VPL];
+      ldg_vec<VPL>(x2, X2 + (int64_t)c * K + col);
+#pragma unroll
+      for (int e = 0; e < VPL; ++e) x[e] *= x2[e];
+    }
+  };
+  int p = p0;
+  for (; p + U <= p1; p += U) {  // full batches
+    advance(p);
+    int c[U];
+    float v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      c[u] = __ldg(crd + p + u);
+      v[u] = __ldg(vals + p + u);
+    }
+    float x[U][VPL];
+#pragma unroll
+    for (int u = 0; u < U; ++u) row(x[u], c[u]);
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v[u], x[u][e], acc[e]);
+  }
+  if (p < p1) {  // the last, partial batch (all its loads still in flight together)
+    advance(p);
     int c[U];
     float v[U];
 #pragma unroll
@@ -290,17 +324,7 @@ __device__ __forceinline__ void gather_pf(float (&acc)[VPL], const int32_t* __re
     float x[U][VPL];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (c[u] >= 0) {
-        ldg_vec<VPL>(x[u], X + (int64_t)c[u] * K + col);
-        if constexpr (H) {
-          float x2[VPL];
-          ldg_vec<VPL>(x2, X2 + (int64_t)c[u] * K + col);
-#pragma unroll
-          for (int e = 0; e < VPL; ++e) x[u][e] *= x2[e];
-        }
-      } else {
-        zero_vec(x[u]);
-      }
+      if (c[u] >= 0) row(x[u], c[u]); else zero_vec(x[u]);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u)
@@ -518,6 +542,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (rec.x >= 0) {
           if constexpr (PF)
             gather_pf<K, VPL, UG, SLNR_TC_PF_AHEAD, H>(acc[0], crd, vals, rec.y, rec.z, X, X2, col, lane % PL::GS);
+          else if constexpr (SLNR_TC_TAIL_BATCH)
+            gather_pf<K, VPL, UG, 0, H>(acc[0], crd, vals, rec.y, rec.z, X, X2, col, lane % PL::GS);
           else
             gather_acc<VPL, UG, H>(acc[0], crd, vals, rec.y, rec.z, X, K, col, X2);
         }
