@@ -346,15 +346,18 @@ def main():
     ap.add_argument("--ref-gflop-per-expr", type=float, default=1.0)
     ap.add_argument("--expr", default="", help="only the expressions whose name contains this (profiling)")
     ap.add_argument("--scale", type=float, default=1.0, help="shrink the workloads (profiling captures)")
-    ap.add_argument("--suite", choices=["main", "next"], default="main",
+    ap.add_argument("--suite", choices=["main", "next", "sweep"], default="main",
                     help="main: the four benchmark expressions (the step); next: <SDDMM,SpMM,GEMM>, "
-                         "<MTTKRP,GEMM>, <SpMMH,GEMM> at full size")
+                         "<MTTKRP,GEMM>, <SpMMH,GEMM> at full size; sweep: <SpMM,GEMM> fused and unfused "
+                         "over the inner dimensions K, L (Sec. 6.3)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.suite == "sweep":
+        return run_sweep(args, rank, world, local)
 
     import torch
 
@@ -492,6 +495,76 @@ def main():
         print(json.dumps(line))
     if pg is not None:
         pg.destroy_process_group()
+    return 0
+
+
+SWEEP_DIMS = (16, 32, 64, 128, 256)
+
+
+def run_sweep(args, rank, world, local):
+    """Sec. 6.3's case study on GB300: <SpMM,GEMM> on the 2^20-vertex R-MAT
+    graph of the benchmark (16 nonzeros per row) for every inner-dimension
+    pair K, L in SWEEP_DIMS, fused and unfused (TF32 allowed), kernel time per
+    call (median, L2 flushed before each).  C (n x K) and D (K x L) are N(0,1)
+    from a seed derived from K and L; the graph is generated once."""
+    import torch
+
+    import paper_2205_11622_gb300 as slnr
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    slnr.build()
+    slnr.lib()
+    n = int((1 << 20) * args.scale)
+    seed = wl.SEED_BASE + 2
+    base = wl.spmm_gemm_rmat(seed, n, 16, 16, 16)
+    B = slnr.DeviceCSR.from_host(base.B, dev)
+    flush = torch.empty(2 * torch.cuda.get_device_properties(dev).L2_cache_size, dtype=torch.uint8, device=dev)
+    ws = slnr.Workspace(device=dev)
+    stream = torch.cuda.current_stream()
+    grid, t0 = [], time.time()
+    for K in SWEEP_DIMS:
+        rk = wl.Rng(seed ^ (K << 20))
+        C = torch.from_numpy(wl.normal(rk, (n, K))).to(dev)
+        for L in SWEEP_DIMS:
+            rl = wl.Rng(seed ^ (K << 20) ^ (L << 8) ^ 1)
+            D = torch.from_numpy(wl.normal(rl, (K, L))).to(dev)
+            w = wl.Workload(f"spmm_gemm_rmat_k{K}_l{L}", "spmm_gemm", base.B, {}, {"K": K, "L": L})
+            out = torch.empty((n, L), dtype=torch.float32, device=dev)
+            res = {"K": K, "L": L, "useful_flops": useful_flops(w), "min_bytes": min_bytes(w)}
+            for variant in ("fused", "unfused"):
+                slnr.spmm_gemm(B, C, D, out=out, variant=variant, workspace=ws)
+                ts = []
+                for it in range(args.warmup + args.steps):
+                    flush.fill_(it & 0xFF)
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    slnr.spmm_gemm(B, C, D, out=out, variant=variant, workspace=ws)
+                    b.record(stream)
+                    b.synchronize()
+                    if it >= args.warmup:
+                        ts.append(a.elapsed_time(b))
+                res[f"{variant}_ms"] = round(statistics.median(ts), 4)
+            if slnr.device_flags() != 0:
+                raise SystemExit(f"device flags {slnr.device_flags():#x} at K={K}, L={L}")
+            res["unfused_over_fused"] = round(res["unfused_ms"] / res["fused_ms"], 3)
+            res["fused_gflops"] = round(res["useful_flops"] / res["fused_ms"] / 1e6, 1)
+            res["fused_hbm_frac"] = round(res["min_bytes"] / res["fused_ms"] / 1e6 / measured_peaks()[0], 4)
+            grid.append(res)
+            del out, D
+        del C
+    best = max(grid, key=lambda r: r["unfused_over_fused"])
+    line = {
+        "metric": "<SpMM,GEMM> unfused/fused time ratio over the inner dimensions (Sec. 6.3)",
+        "value": round(statistics.geometric_mean(r["unfused_over_fused"] for r in grid), 3), "unit": "x (geomean)",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "n/a",
+        "vs_baseline": None, "dtype": "f32 (tf32 tensor-core contractions allowed)", "data": "synthetic",
+        "config": {"workload": f"spmm_gemm R-MAT {n}x{n}, 16 nnz/row (seed {seed:#x}), K, L in {list(SWEEP_DIMS)}",
+                   "l2": "flushed before every call", "timing": "median kernel time per call, CUDA events"},
+        "best": {"K": best["K"], "L": best["L"], "unfused_over_fused": best["unfused_over_fused"]},
+        "grid": grid, "seconds": round(time.time() - t0, 1),
+    }
+    if rank == 0:
+        print(json.dumps(line))
     return 0
 
 
