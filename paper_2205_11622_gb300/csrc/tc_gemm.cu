@@ -202,16 +202,25 @@ __device__ __forceinline__ int mbar_wait_or_end(uint64_t* bar, uint32_t parity, 
 // X[k,:] .* X2[k,:] (<SpMMH,GEMM>); kDense: rows of a materialised T.
 enum TcMode { kSegments = 0, kDense = 1, kSegmentsH = 2 };
 
+// Columns of the T tile and of D^T: K, padded to one 128-byte swizzle atom
+// (32 tf32 values) when K = 16; the padding columns hold zeros.
+__host__ __device__ constexpr int tc_kt(int K) { return K < 32 ? 32 : K; }
+
 // Number of T / accumulator buffers: up to four, as many as fit beside D^T
 // in shared memory (200 KB budget) and in tensor memory (512 columns).
 __host__ __device__ constexpr int tc_nbuf(int K, int L) {
-  return ((size_t)4 * kTcRows * K * 4 + (size_t)L * K * 4 + 1024 <= (size_t)200 * 1024 && 4 * L <= 512) ? 4 : 2;
+  return ((size_t)4 * kTcRows * tc_kt(K) * 4 + (size_t)L * tc_kt(K) * 4 + 1024 <= (size_t)200 * 1024 && 4 * L <= 512)
+             ? 4
+             : ((size_t)2 * kTcRows * tc_kt(K) * 4 + (size_t)L * tc_kt(K) * 4 + 1024 <= (size_t)200 * 1024 &&
+                2 * L <= 512)
+                   ? 2
+                   : 1;
 }
 
-// Shared memory: NBUF T tiles (kTcRows x K) and D^T (L x K), tf32 K-major
+// Shared memory: NBUF T tiles (kTcRows x KT) and D^T (L x KT), tf32 K-major
 // 128B-swizzled, plus 1 KB of alignment slack.
 __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
-  return (size_t)tc_nbuf(K, L) * kTcRows * K * 4 + (size_t)L * K * 4 + 1024;
+  return (size_t)tc_nbuf(K, L) * kTcRows * tc_kt(K) * 4 + (size_t)L * tc_kt(K) * 4 + 1024;
 }
 
 #ifndef SLNR_TC_VPL
@@ -251,7 +260,7 @@ __device__ __forceinline__ void gather_pf(float (&acc)[VPL], const int32_t* __re
                                           const float* __restrict__ vals, int p0, int p1,
                                           const float* __restrict__ X, const float* __restrict__ X2, int col,
                                           int gl) {
-  constexpr int GS = K / VPL, LPR = K / 32, RPI = GS / LPR;
+  constexpr int GS = K / VPL, LPR = K >= 32 ? K / 32 : 1, RPI = GS / LPR;  // a row of 16 floats is half a line
   static_assert(AHEAD % RPI == 0, "the prefetch window is whole steps");
   constexpr int NPF = AHEAD / RPI;
   const int prow = gl / LPR, poff = (gl % LPR) * 32;
@@ -392,14 +401,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ D,
               float* __restrict__ A,
               float* __restrict__ partial) {
-  static_assert(K % 32 == 0 && K >= 32 && K <= 128, "K must be 32, 64 or 128");
-  static_assert(L % 32 == 0 && L >= 32 && L <= 256, "L must be a multiple of 32 in [32, 256]");
+  static_assert(K == 16 || K == 32 || K == 64 || K == 128, "K must be 16, 32, 64 or 128");
+  static_assert(L % 16 == 0 && L >= 16 && L <= 256, "L must be a multiple of 16 in [16, 256]");
+  constexpr int KT = tc_kt(K);  // tile columns (K, or 32 with zero padding)
   static_assert(kTcThreads == 1024, "32 warps: 27 producers, 1 MMA, 4 epilogue");
   using PL = ProdLayout<K>;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
   constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
-  constexpr int TBYTES = kTcRows * K * 4;
+  constexpr int TBYTES = kTcRows * KT * 4;
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t full_bar[NBUF], mma_bar[NBUF], free_bar[NBUF];
   __shared__ int2 dest[NBUF][kTcRows];  // per slot: (A row, partial slot); x < 0 = padding
@@ -450,14 +460,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tile_seq[0] = 1;
     end_tile = g0 >= ntiles ? 0 : INT_MAX;
   }
-  // D (K x L, row-major) -> D^T as the B operand (L rows of K), tf32
-  for (int i = tid; i < K * (L / 4); i += kTcThreads) {
+  // D (K x L, row-major) -> D^T as the B operand (L rows of KT), tf32; rows
+  // k >= K of the padded tile are zero
+  for (int i = tid; i < KT * (L / 4); i += kTcThreads) {
     const int k = i / (L / 4), n4 = i % (L / 4);
-    const float4 d = __ldg(reinterpret_cast<const float4*>(D + (int64_t)k * L) + n4);
+    const float4 d = k < K ? __ldg(reinterpret_cast<const float4*>(D + (int64_t)k * L) + n4)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
     const float dv[4] = {d.x, d.y, d.z, d.w};
 #pragma unroll
     for (int e = 0; e < 4; ++e)
       *reinterpret_cast<uint32_t*>(sD + tc::sw128_offset(4 * n4 + e, k, L)) = tc::to_tf32(dv[e]);
+  }
+  if constexpr (KT > K) {  // the padding columns of every T buffer: zero once, never written
+    for (int i = tid; i < NBUF * kTcRows * (KT - K); i += kTcThreads) {
+      const int b = i / (kTcRows * (KT - K)), r = (i / (KT - K)) % kTcRows, k = K + i % (KT - K);
+      *reinterpret_cast<uint32_t*>(sT + b * TBYTES + tc::sw128_offset(r, k, kTcRows)) = 0u;
+    }
   }
   tc::fence_proxy_async_smem();
   tc::tc_fence_before_sync();
@@ -603,7 +621,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tc::tc_fence_after_sync();
         const uint32_t a_base = sT_addr + b * TBYTES;
 #pragma unroll
-        for (int kb = 0; kb < K / 32; ++kb)
+        for (int kb = 0; kb < KT / 32; ++kb)
 #pragma unroll
           for (int ks = 0; ks < 4; ++ks) {
             const uint64_t ad = tc::desc_k_sw128(a_base + kb * kTcRows * 128 + ks * 32);
@@ -634,14 +652,24 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (q == 0 && lane == 0) tc::st_release_smem(&mma_tiles_done, j + 1);
       float* dst = nullptr;
       if (dd.x >= 0) dst = dd.y < 0 ? A + (int64_t)dd.x * L : partial + (int64_t)dd.y * L;
+      if constexpr (L >= 32) {
 #pragma unroll 1
-      for (int c = 0; c < L; c += 32) {
-        float v[32];
-        tc::tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
-        if (dst != nullptr) {
-          float4* o = reinterpret_cast<float4*>(dst + c);
+        for (int c = 0; c < L; c += 32) {
+          float v[32];
+          tc::tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
+          if (dst != nullptr) {
+            float4* o = reinterpret_cast<float4*>(dst + c);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          }
+        }
+      } else {
+        float v[16];
+        tc::tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L), v);
+        if (dst != nullptr) {
+          float4* o = reinterpret_cast<float4*>(dst);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
       }
       tc::tc_fence_before_sync();
@@ -726,9 +754,10 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
                                                                              X2, D, A, partial);          \
     return cudaGetLastError();                                                                            \
   }
-  SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
-  SLNR_TC_CASE(64, 32) SLNR_TC_CASE(64, 64) SLNR_TC_CASE(64, 128) SLNR_TC_CASE(64, 256)
-  SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128)
+  SLNR_TC_CASE(16, 16) SLNR_TC_CASE(16, 32) SLNR_TC_CASE(16, 64) SLNR_TC_CASE(16, 128) SLNR_TC_CASE(16, 256)
+  SLNR_TC_CASE(32, 16) SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
+  SLNR_TC_CASE(64, 16) SLNR_TC_CASE(64, 32) SLNR_TC_CASE(64, 64) SLNR_TC_CASE(64, 128) SLNR_TC_CASE(64, 256)
+  SLNR_TC_CASE(128, 16) SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128) SLNR_TC_CASE(128, 256)
 #undef SLNR_TC_CASE
   return cudaErrorInvalidValue;
 }
@@ -749,7 +778,7 @@ size_t l2_bytes() {
 }  // namespace
 
 bool tc_supported(int K, int L) {
-  return (K == 32 || K == 64 || K == 128) && (L == 32 || L == 64 || L == 128 || L == 256) &&
+  return (K == 16 || K == 32 || K == 64 || K == 128) && (L == 16 || L == 32 || L == 64 || L == 128 || L == 256) &&
          tc_smem_bytes(K, L) <= (size_t)200 * 1024;
 }
 

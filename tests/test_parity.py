@@ -56,8 +56,8 @@ def test_small_workloads(slnr, orc, idx, variant, allow_tf32):
     check(slnr, orc, wl.small(idx), variant, allow_tf32)
 
 
-@pytest.mark.parametrize("K,L", [(4, 8), (8, 4), (16, 256), (256, 16), (32, 32), (64, 128), (128, 64), (128, 128),
-                                 (256, 256)])
+@pytest.mark.parametrize("K,L", [(4, 8), (8, 4), (16, 16), (16, 256), (64, 16), (256, 16), (32, 32), (64, 128),
+                                 (128, 64), (128, 128), (128, 256), (256, 256)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_spmm_gemm_widths(slnr, orc, K, L, variant):
     w = wl.spmm_gemm_rmat(0x51A4 + 7 * K + L, 1537, 12, K, L)
@@ -79,7 +79,8 @@ def test_mttkrp_widths(slnr, orc, L, variant):
     check(slnr, orc, w, variant)
 
 
-@pytest.mark.parametrize("L,M", [(4, 16), (16, 4), (32, 64), (64, 64), (128, 32), (256, 128)])
+@pytest.mark.parametrize("L,M", [(4, 16), (16, 4), (16, 16), (16, 64), (32, 16), (32, 64), (64, 64), (128, 32),
+                                 (128, 256), (256, 128)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_spttm_ttm_widths(slnr, orc, L, M, variant):
     w = wl.spttm_ttm_powerlaw(0x51A4 + L + M, (60, 70, 900), 12000, 8.0, 900, L, M)
