@@ -14,6 +14,13 @@
 // (spmm.cu over the fiber level), then k_mttkrp_stage2_units reads it.
 #include "launch.h"
 
+#ifndef SLNR_MTTKRP_MIN_CTAS
+#define SLNR_MTTKRP_MIN_CTAS 5  // resident 256-thread CTAs per SM the unit kernel is compiled for (48 registers)
+#endif
+#ifndef SLNR_MTTKRP_U
+#define SLNR_MTTKRP_U 4  // nonzeros of a fiber in flight per lane group
+#endif
+
 namespace slnr {
 namespace {
 
@@ -38,7 +45,7 @@ __device__ __forceinline__ void unit_fibers(const Unit un, const SliceUnits su, 
 }
 
 template <int L>
-__global__ void __launch_bounds__(256) k_mttkrp_units(const WsHeader* __restrict__ hdr,
+__global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(const WsHeader* __restrict__ hdr,
                                                       const Unit* __restrict__ units,
                                                       const SliceUnits* __restrict__ sus, int max_units,
                                                       const int32_t* __restrict__ pos2,
@@ -67,7 +74,7 @@ __global__ void __launch_bounds__(256) k_mttkrp_units(const WsHeader* __restrict
       // producer: T(l) = sum_k B(i,j,k) D(k,l), in registers
       float t[RL::VPL];
       zero_vec(t);
-      gather_acc<RL::VPL>(t, crd3, vals, p0, p1, D, L, col);
+      gather_acc<RL::VPL, SLNR_MTTKRP_U>(t, crd3, vals, p0, p1, D, L, col);
       // consumer: A(i,l) += T(l) C(j,l)
 #pragma unroll
       for (int x = 0; x < RL::VPL; ++x) acc[x] = fmaf(t[x], c[x], acc[x]);

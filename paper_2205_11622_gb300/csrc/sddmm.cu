@@ -14,6 +14,13 @@
 #include "launch.h"
 #include "tile.cuh"
 
+#ifndef SLNR_SDDMM_MIN_CTAS
+#define SLNR_SDDMM_MIN_CTAS 4  // resident 256-thread CTAs per SM the fused kernels are compiled for (64 registers)
+#endif
+#ifndef SLNR_SDDMM_U
+#define SLNR_SDDMM_U 2  // nonzeros in flight per lane group
+#endif
+
 namespace slnr {
 namespace {
 
@@ -22,7 +29,7 @@ namespace {
 //   acc += vals[p] * <c, D(crd[p], :)> * E(crd[p], :)
 // Every lane of the warp runs the same number of steps (shuffles stay
 // converged); lanes past the end use zero weights and load nothing.
-template <int WM, int U = 2>
+template <int WM, int U = SLNR_SDDMM_U>
 __device__ __forceinline__ void sddmm_spmm_range(float (&acc)[RowLanes<WM>::VPL],
                                                  const float (&c)[RowLanes<WM>::VPL], int p0, int p1,
                                                  const int32_t* __restrict__ crd,
@@ -63,7 +70,7 @@ __device__ __forceinline__ void sddmm_spmm_range(float (&acc)[RowLanes<WM>::VPL]
 }
 
 template <int WM>
-__global__ void __launch_bounds__(256) k_sddmm_spmm_rows(int nrows, const int32_t* __restrict__ pos,
+__global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_rows(int nrows, const int32_t* __restrict__ pos,
                                                          const int32_t* __restrict__ crd,
                                                          const float* __restrict__ vals,
                                                          const float* __restrict__ C,
@@ -87,7 +94,7 @@ __global__ void __launch_bounds__(256) k_sddmm_spmm_rows(int nrows, const int32_
 }
 
 template <int WM>
-__global__ void __launch_bounds__(256) k_sddmm_spmm_chunks(const WsHeader* __restrict__ hdr,
+__global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_chunks(const WsHeader* __restrict__ hdr,
                                                            const Chunk* __restrict__ chunks, int max_chunks,
                                                            const int32_t* __restrict__ crd,
                                                            const float* __restrict__ vals,
@@ -118,7 +125,7 @@ __global__ void __launch_bounds__(256) k_sddmm_spmm_chunks(const WsHeader* __res
 // multiplied by W (LW x M) and A's rows are written once.  Rows with more than
 // kLightMax nonzeros are left to the chunk kernel and k_combine (times W).
 template <int WM, int LW>
-__global__ void __launch_bounds__(256) k_sddmm_spmm_gemm_tiles(int nrows, const int32_t* __restrict__ pos,
+__global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_gemm_tiles(int nrows, const int32_t* __restrict__ pos,
                                                                const int32_t* __restrict__ crd,
                                                                const float* __restrict__ vals,
                                                                const float* __restrict__ C,
