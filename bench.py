@@ -391,10 +391,11 @@ def main():
     wspaces = [slnr.Workspace(device=dev) for _ in ws]
     outs = [None] * len(ws)
 
-    def call(i, out=None):
+    def call(i, out=None, on_stream=None):
         w = ws[i]
         B, dense = dev_inputs[i]
-        return slnr.run(w.op, B, dense, out=out, variant=args.variant, allow_tf32=allow_tf32, workspace=wspaces[i])
+        return slnr.run(w.op, B, dense, out=out, variant=args.variant, allow_tf32=allow_tf32, workspace=wspaces[i],
+                        stream=on_stream)
 
     for i in range(len(ws)):
         outs[i] = call(i)
@@ -570,30 +571,55 @@ def run_sweep(args, rank, world, local):
 
 def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_flops, world, pg, dev):
     """Same step through the public API with host buffers: every step copies all
-    inputs from pinned host memory to the device and all outputs back."""
-    host_in, dev_in, host_out, dev_out = [], [], [], []
+    inputs from pinned host memory to the device and all outputs back.  The
+    copies run on two streams of their own (host-to-device and device-to-host,
+    both directions of the link at once) and overlap the calls of the other
+    expressions: expression i computes once its inputs have arrived and its
+    previous outputs have been read back, and its outputs are copied out as
+    soon as it is done; a step's inputs overwrite the device buffers only
+    after the previous step's call that reads them has finished."""
+    n = len(ws)
+    host_in, dev_in, host_out, dev_out = [[] for _ in range(n)], [[] for _ in range(n)], [[] for _ in range(n)], \
+        [[] for _ in range(n)]
     for i, w in enumerate(ws):
         B, dense = dev_inputs[i]
         arrays = [getattr(B, f) for f in ("pos", "crd", "vals")] if w.op in CSR_OPS else \
             [getattr(B, f) for f in ("pos1", "crd1", "pos2", "crd2", "pos3", "crd3", "vals")]
         arrays += list(dense.values())
         for a in arrays:
-            dev_in.append(a)
-            host_in.append(a.cpu().pin_memory())
+            dev_in[i].append(a)
+            host_in[i].append(a.cpu().pin_memory())
         o = outs[i]
         for t in (o if isinstance(o, tuple) else (o,)):
-            dev_out.append(t)
-            host_out.append(torch.empty(t.shape, dtype=t.dtype, pin_memory=True))
-    h2d = sum(t.numel() * t.element_size() for t in host_in)
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
+            dev_out[i].append(t)
+            host_out[i].append(torch.empty(t.shape, dtype=t.dtype, pin_memory=True))
+    h2d = sum(t.numel() * t.element_size() for hs in host_in for t in hs)
+    d2h = sum(t.numel() * t.element_size() for hs in host_out for t in hs)
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    in_ready = [torch.cuda.Event() for _ in range(n)]
+    done = [torch.cuda.Event() for _ in range(n)]
+    read_back = [torch.cuda.Event() for _ in range(n)]
+    for i in range(n):  # nothing pending before the first step
+        done[i].record(stream)
+        read_back[i].record(stream)
 
     def step():
-        for d, h in zip(dev_in, host_in):
-            d.copy_(h, non_blocking=True)
-        for i in range(len(ws)):
-            call(i, out=outs[i])
-        for h, d in zip(host_out, dev_out):
-            h.copy_(d, non_blocking=True)
+        for i in range(n):
+            s_in.wait_event(done[i])            # the previous call reading these inputs has finished
+            with torch.cuda.stream(s_in):
+                for d, h in zip(dev_in[i], host_in[i]):
+                    d.copy_(h, non_blocking=True)
+            in_ready[i].record(s_in)
+        for i in range(n):
+            stream.wait_event(in_ready[i])
+            stream.wait_event(read_back[i])     # the previous outputs have been read back
+            call(i, out=outs[i], on_stream=stream)
+            done[i].record(stream)
+            s_out.wait_event(done[i])
+            with torch.cuda.stream(s_out):
+                for h, d in zip(host_out[i], dev_out[i]):
+                    h.copy_(d, non_blocking=True)
+            read_back[i].record(s_out)
 
     for _ in range(2):
         step()
@@ -602,8 +628,12 @@ def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_fl
         pg.barrier()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record(stream)
+    s_in.wait_stream(stream)
+    s_out.wait_stream(stream)
     for _ in range(steps):
         step()
+    stream.wait_stream(s_in)
+    stream.wait_stream(s_out)
     b.record(stream)
     b.synchronize()
     ms = a.elapsed_time(b) / steps
@@ -612,7 +642,8 @@ def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_fl
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
         ms = float(t.item())
     return {"value": round(world * total_flops / (ms / 1e3) / 1e9, 2), "unit": "GFLOP/s",
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 3)}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 3),
+            "link_gbs": round((h2d + d2h) / (ms / 1e3) / 1e9, 1)}
 
 
 if __name__ == "__main__":
