@@ -241,6 +241,9 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 #ifndef SLNR_TC_TAIL_BATCH
 #define SLNR_TC_TAIL_BATCH 1  // segments without prefetch: the last batch loaded at once (0: row by row)
 #endif
+#ifndef SLNR_TC_SEQ_SEGS
+#define SLNR_TC_SEQ_SEGS 2  // segments a lane group claims at once and gathers one after the other
+#endif
 #ifndef SLNR_TC_PF_AHEAD
 #define SLNR_TC_PF_AHEAD 8  // rows of a segment prefetched into L2 beyond the batch in flight
 #endif
@@ -383,11 +386,11 @@ __device__ __forceinline__ void store_t_part(uint8_t* sTb, int s, int col, const
 // completed tiles that the epilogue publishes (release) once all four
 // epilogue warps have read the tile's row destinations.  Every wait is
 // bounded; a timeout raises kErrTimeout and the CTA winds down.
-// Items per producer claim: one per lane group (a segment), or
-// SLNR_TC_DENSE_ROWS per lane group in DENSE mode.
+// Items per producer claim: SLNR_TC_SEQ_SEGS segments per lane group, or
+// SLNR_TC_DENSE_ROWS rows per lane group in DENSE mode.
 template <int K, int MODE>
 __host__ __device__ constexpr int claim_items() {
-  return ProdLayout<K>::G * (MODE == kDense ? SLNR_TC_DENSE_ROWS : 1);
+  return ProdLayout<K>::G * (MODE == kDense ? SLNR_TC_DENSE_ROWS : SLNR_TC_SEQ_SEGS);
 }
 
 constexpr int kProducerWarps = 27;
@@ -512,7 +515,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // then waits for its buffer to be free (the MMAs of tile c / CPT - NBUF
     // completed and their destinations read), stores the rows and their
     // destinations, and lane 0 arrives once for the claim.
-    constexpr int VPL = PL::VPL, G = PL::G, R = MODE != kDense ? 1 : SLNR_TC_DENSE_ROWS;
+    constexpr int VPL = PL::VPL, G = PL::G, R = MODE != kDense ? SLNR_TC_SEQ_SEGS : SLNR_TC_DENSE_ROWS;
     constexpr int IPC = G * R, CPT = kTcRows / IPC;
     static_assert(IPC == claim_items<K, MODE>(), "barrier count matches the claims");
     static_assert(kTcRows % IPC == 0, "claims tile the item tile");
@@ -553,19 +556,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       float acc[R][VPL];
       int2 dst0 = make_int2(-1, -1);  // destination of the segment (R = 1)
       if constexpr (MODE != kDense) {
+        // the group's R segments, one after the other (the first record was
+        // loaded with the previous claim; the others share its cache line)
+        int4 rr[R];
+        rr[0] = rec;
+#pragma unroll
+        for (int r = 1; r < R; ++r) rr[r] = load_rec(gid, cl, r);
         const int4 rec_next = gid_next >= 0 ? load_rec(gid_next, cl_next, 0) : make_int4(-1, 0, 0, -1);
-        zero_vec(acc[0]);
         constexpr bool H = MODE == kSegmentsH;
         constexpr int UG = H ? PL::U / 2 : PL::U;  // two loads per nonzero in Hadamard mode
-        if (rec.x >= 0) {
-          if constexpr (PF)
-            gather_pf<K, VPL, UG, SLNR_TC_PF_AHEAD, H>(acc[0], crd, vals, rec.y, rec.z, X, X2, col, lane % PL::GS);
-          else if constexpr (SLNR_TC_TAIL_BATCH)
-            gather_pf<K, VPL, UG, 0, H>(acc[0], crd, vals, rec.y, rec.z, X, X2, col, lane % PL::GS);
-          else
-            gather_acc<VPL, UG, H>(acc[0], crd, vals, rec.y, rec.z, X, K, col, X2);
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          zero_vec(acc[r]);
+          if (rr[r].x >= 0) {
+            if constexpr (PF)
+              gather_pf<K, VPL, UG, SLNR_TC_PF_AHEAD, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, X2, col,
+                                                          lane % PL::GS);
+            else if constexpr (SLNR_TC_TAIL_BATCH)
+              gather_pf<K, VPL, UG, 0, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, X2, col, lane % PL::GS);
+            else
+              gather_acc<VPL, UG, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, K, col, X2);
+          }
         }
-        dst0 = make_int2(rec.x, rec.w);
+        dst0 = make_int2(rr[0].x, rr[0].w);
         rec = rec_next;
       } else {
 #pragma unroll
@@ -592,8 +605,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         store_t_part<VPL>(sT + b * TBYTES, s0 + r * G, col, acc[r]);
-        if (lane % PL::GS == 0)
-          dest[b][s0 + r * G] = MODE != kDense ? dst0 : make_int2(load_rec(gid, cl, r).x, -1);
+        if (lane % PL::GS == 0) {
+          if constexpr (MODE == kDense) {
+            dest[b][s0 + r * G] = make_int2(load_rec(gid, cl, r).x, -1);
+          } else if (r == 0) {
+            dest[b][s0] = dst0;
+          } else {
+            const int4 rq = load_rec(gid, cl, r);
+            dest[b][s0 + r * G] = make_int2(rq.x, rq.w);
+          }
+        }
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
