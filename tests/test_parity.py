@@ -240,3 +240,13 @@ def test_gathered_matrix_larger_than_l2(slnr, orc, K, L):
     # uniform columns give partial last batches in every row
     w = wl.spmm_gemm_uniform(0x51A4 + K + L, 3001, 1 << 20, 21, K, L, name=f"spmm_gemm_wide_{K}")
     check(slnr, orc, w, "fused", True)
+
+
+@pytest.mark.parametrize("K,L", [(16, 16), (32, 64), (128, 128), (128, 256)])
+@pytest.mark.parametrize("nrows", [1, 3, 130])
+def test_tensor_core_path_on_tiny_inputs(slnr, orc, K, L, nrows):
+    # fewer rows than one 128-row tile, exactly one tile plus a ragged second:
+    # the dynamic tile counter hands out one or two tiles to a full grid of CTAs
+    w = wl.spmm_gemm_uniform(0x51A4 + 13 * K + L + nrows, nrows, 300, 7, K, L, name=f"tiny_{nrows}")
+    check(slnr, orc, w, "fused", True)
+    check(slnr, orc, w, "unfused", True)
