@@ -55,9 +55,11 @@ struct SliceUnits {      // MTTKRP: units of one slice
   int count;
 };
 
-struct Unit {            // MTTKRP: window `u` of slice `slice`
+struct Unit {            // MTTKRP: window `u` of slice `slice`, fibers [flo, fhi)
   int slice;
   int u;
+  int flo;
+  int fhi;
 };
 
 // Validation flag bits

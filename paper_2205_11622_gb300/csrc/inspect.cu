@@ -48,20 +48,56 @@ __global__ void k_classify(int nrows, const int32_t* __restrict__ pos, WsHeader*
   }
 }
 
+// First f in [lo, hi) with pos[f] >= key (hi if none).
+__device__ __forceinline__ int lower_bound_pos(const int32_t* __restrict__ pos, int lo, int hi, int key) {
+  while (lo < hi) {
+    const int mid = lo + ((hi - lo) >> 1);
+    if (__ldg(pos + mid) < key) lo = mid + 1; else hi = mid;
+  }
+  return lo;
+}
+
+// One warp per slice: the slice is cut into units, the fibers that start in
+// one window of kUnitNnz nonzeros, and the lanes write the unit records.
 __global__ void k_csf_units(int nslices, const int32_t* __restrict__ pos2,
                             const int32_t* __restrict__ pos3, WsHeader* hdr,
                             SliceUnits* __restrict__ su, Unit* __restrict__ units, int max_units) {
-  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < nslices; s += gridDim.x * blockDim.x) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t sw = warp; sw < nslices; sw += nwarps) {
+    const int s = (int)sw;
     const int n = pos3[pos2[s + 1]] - pos3[pos2[s]];
     const int nu = n > 0 ? (n + kUnitNnz - 1) / kUnitNnz : 1;
-    const int base = atomicAdd(&hdr->n_units, nu);
+    int base = 0;
+    if (lane == 0) base = atomicAdd(&hdr->n_units, nu);
+    base = __shfl_sync(0xffffffffu, base, 0);
     if (base + nu > max_units) {
-      atomicOr(&hdr->error, kErrOverflow);
-      su[s] = SliceUnits{0, 0};
+      if (lane == 0) {
+        atomicOr(&hdr->error, kErrOverflow);
+        su[s] = SliceUnits{0, 0};
+      }
       continue;
     }
-    su[s] = SliceUnits{base, nu};
-    for (int u = 0; u < nu; ++u) units[base + u] = Unit{s, u};
+    if (lane == 0) su[s] = SliceUnits{base, nu};
+    for (int u = lane; u < nu; u += 32) units[base + u] = Unit{s, u, 0, 0};
+  }
+}
+
+// One thread per unit: its fiber range [flo, fhi), the fibers of its slice
+// whose first nonzero lies in the unit's window (binary searches over pos3).
+__global__ void k_unit_ranges(const WsHeader* __restrict__ hdr, int max_units, const int32_t* __restrict__ pos2,
+                              const int32_t* __restrict__ pos3, const SliceUnits* __restrict__ su,
+                              Unit* __restrict__ units) {
+  const int n = min(hdr->n_units, max_units);
+  for (int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; w < n; w += (int64_t)gridDim.x * blockDim.x) {
+    Unit un = units[w];
+    const int f0 = pos2[un.slice], f1 = pos2[un.slice + 1];
+    const int start = pos3[f0], count = su[un.slice].count;
+    const int lo_key = start + un.u * kUnitNnz;
+    un.flo = un.u == 0 ? f0 : lower_bound_pos(pos3, f0, f1, lo_key);
+    un.fhi = un.u == count - 1 ? f1 : lower_bound_pos(pos3, f0, f1, lo_key + kUnitNnz);
+    units[w] = un;
   }
 }
 
@@ -127,8 +163,10 @@ cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_
 
 cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s) {
   if (B.nslices <= 0) return cudaSuccess;
-  k_csf_units<<<grid_for(B.nslices, 256), 256, 0, s>>>(B.nslices, B.pos2, B.pos3, plan.hdr,
-                                                       plan.slice_units, plan.units, plan.max_units);
+  k_csf_units<<<grid_for((int64_t)B.nslices * 32, 256), 256, 0, s>>>(B.nslices, B.pos2, B.pos3, plan.hdr,
+                                                                     plan.slice_units, plan.units, plan.max_units);
+  k_unit_ranges<<<grid_for(plan.max_units, 256), 256, 0, s>>>(plan.hdr, plan.max_units, B.pos2, B.pos3,
+                                                               plan.slice_units, plan.units);
   return cudaGetLastError();
 }
 

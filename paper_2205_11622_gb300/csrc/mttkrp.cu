@@ -24,26 +24,6 @@
 namespace slnr {
 namespace {
 
-// First f in [lo, hi) with pos[f] >= key (hi if none).
-__device__ __forceinline__ int lower_bound_pos(const int32_t* __restrict__ pos, int lo, int hi, int key) {
-  while (lo < hi) {
-    const int mid = lo + ((hi - lo) >> 1);
-    if (__ldg(pos + mid) < key) lo = mid + 1; else hi = mid;
-  }
-  return lo;
-}
-
-// Fiber range [*flo, *fhi) of unit un: the fibers of its slice whose first
-// nonzero lies in the unit's window of kUnitNnz nonzeros.
-__device__ __forceinline__ void unit_fibers(const Unit un, const SliceUnits su, const int32_t* __restrict__ pos2,
-                                            const int32_t* __restrict__ pos3, int* flo, int* fhi) {
-  const int f0 = __ldg(pos2 + un.slice), f1 = __ldg(pos2 + un.slice + 1);
-  const int start = __ldg(pos3 + f0);
-  const int lo_key = start + un.u * kUnitNnz;
-  *flo = un.u == 0 ? f0 : lower_bound_pos(pos3, f0, f1, lo_key);
-  *fhi = un.u == su.count - 1 ? f1 : lower_bound_pos(pos3, f0, f1, lo_key + kUnitNnz);
-}
-
 template <int L>
 __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(const WsHeader* __restrict__ hdr,
                                                       const Unit* __restrict__ units,
@@ -63,8 +43,7 @@ __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(cons
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t w = warp; w < n; w += nwarps) {
     const Unit un = units[w];
-    int flo, fhi;
-    unit_fibers(un, sus[un.slice], pos2, pos3, &flo, &fhi);
+    const int flo = un.flo, fhi = un.fhi;  // fibers starting in the unit's window (inspector)
     float acc[RL::VPL];
     zero_vec(acc);
     for (int f = flo + grp; f < fhi; f += RL::GPW) {
@@ -101,8 +80,7 @@ __global__ void __launch_bounds__(256) k_mttkrp_stage2_units(const WsHeader* __r
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t w = warp; w < n; w += nwarps) {
     const Unit un = units[w];
-    int flo, fhi;
-    unit_fibers(un, sus[un.slice], pos2, pos3, &flo, &fhi);
+    const int flo = un.flo, fhi = un.fhi;  // fibers starting in the unit's window (inspector)
     float acc[RL::VPL];
     zero_vec(acc);
     for (int f = flo + grp; f < fhi; f += RL::GPW) {
@@ -118,13 +96,13 @@ __global__ void __launch_bounds__(256) k_mttkrp_stage2_units(const WsHeader* __r
   }
 }
 
-// One CTA per output row i: find i's slice, sum its units' partials (strided
-// lanes, then a fixed pairwise tree), write A(i,:) (zeros without a slice).
-// With E (L x M, <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and
-// A(i,:) = u(i,:).E is written instead (width M): the MTTKRP result is never
-// stored.
+// One CTA per slice q (grid-stride): sums the slice's unit partials (strided
+// lanes, then a fixed pairwise tree) and writes A(crd1[q], :).  Rows of A
+// without a slice were zero-filled before the launch.  With E (L x M,
+// <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and A(i,:) = u(i,:).E
+// is written instead (width M): the MTTKRP result is never stored.
 template <int L>
-__global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, const int32_t* __restrict__ crd1,
+__global__ void __launch_bounds__(256) k_mttkrp_combine(int nslices, const int32_t* __restrict__ crd1,
                                                         const SliceUnits* __restrict__ sus,
                                                         const float* __restrict__ partial,
                                                         const float* __restrict__ E, int M,
@@ -133,21 +111,12 @@ __global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, con
   constexpr int NR = 256 / NC;
   __shared__ float4 red[256];
   const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
-  for (int i = blockIdx.x; i < d0; i += gridDim.x) {
-    int lo = 0, hi = nslices;  // first slice with crd1 >= i
-    while (lo < hi) {
-      const int mid = lo + ((hi - lo) >> 1);
-      if (__ldg(crd1 + mid) < i) lo = mid + 1; else hi = mid;
-    }
-    int base = 0, count = 0;
-    if (lo < nslices && __ldg(crd1 + lo) == i) {
-      const SliceUnits su = sus[lo];
-      base = su.base;
-      count = su.count;
-    }
+  for (int q = blockIdx.x; q < nslices; q += gridDim.x) {
+    const int i = __ldg(crd1 + q);
+    const SliceUnits su = sus[q];
     float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int u = rl; u < count; u += NR) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(base + u) * L) + c4);
+    for (int u = rl; u < su.count; u += NR) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L) + c4);
       s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
     }
     red[threadIdx.x] = s;
@@ -164,11 +133,11 @@ __global__ void __launch_bounds__(256) k_mttkrp_combine(int d0, int nslices, con
     if (E == nullptr) {
       if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
     } else {
-      const float* u = reinterpret_cast<const float*>(red);  // u(i,0..L)
+      const float* uu = reinterpret_cast<const float*>(red);  // u(i,0..L)
       for (int m = threadIdx.x; m < M; m += blockDim.x) {
         float acc = 0.f;
 #pragma unroll 8
-        for (int l = 0; l < L; ++l) acc = fmaf(u[l], __ldg(E + (int64_t)l * M + m), acc);
+        for (int l = 0; l < L; ++l) acc = fmaf(uu[l], __ldg(E + (int64_t)l * M + m), acc);
         A[(int64_t)i * M + m] = acc;
       }
     }
@@ -209,12 +178,14 @@ cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T
 cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M,
                                   float* A, cudaStream_t s) {
   if (B.dim[0] <= 0) return cudaSuccess;
-  int grid = B.dim[0];
+  // rows of A without a slice are zero; the kernel writes the others
+  cudaError_t e = cudaMemsetAsync(A, 0, sizeof(float) * (size_t)B.dim[0] * (size_t)(E != nullptr ? M : L), s);
+  if (e != cudaSuccess || B.nslices <= 0) return e;
+  int grid = B.nslices;
   const int cap = device_sm_count() * 8;
   if (grid > cap) grid = cap;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.dim[0], B.nslices, B.crd1, plan.slice_units, plan.partial, E, M,
-                                              A);
+    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial, E, M, A);
   });
   return cudaGetLastError();
 }
