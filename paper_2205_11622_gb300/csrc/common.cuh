@@ -32,7 +32,9 @@ struct WsHeader {        // first 256 bytes of every workspace
   int error;             // validation / runtime flags (bit set = problem found)
   int n_segs;            // segments of the tensor-core path
   int next_tile;         // tensor-core path: next item tile to hand to a CTA
-  int pad[58];
+  int next_row;          // fused <SDDMM,SpMM>: next block of rows to hand to a warp
+  int next_unit;         // fused MTTKRP: next unit to hand to a warp
+  int pad[56];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 

@@ -25,7 +25,7 @@ namespace slnr {
 namespace {
 
 template <int L>
-__global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(const WsHeader* __restrict__ hdr,
+__global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(WsHeader* __restrict__ hdr,
                                                       const Unit* __restrict__ units,
                                                       const SliceUnits* __restrict__ sus, int max_units,
                                                       const int32_t* __restrict__ pos2,
@@ -39,9 +39,13 @@ __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(cons
   using RL = RowLanes<L>;
   const int n = min(hdr->n_units, max_units);
   const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t w = warp; w < n; w += nwarps) {
+  // warps take units one at a time from the header's counter (units of hub
+  // slices hold far more work than those of small slices)
+  for (;;) {
+    int w = 0;
+    if (lane == 0) w = atomicAdd(&hdr->next_unit, 1);
+    w = __shfl_sync(0xffffffffu, w, 0);
+    if (w >= n) break;
     const Unit un = units[w];
     const int flo = un.flo, fhi = un.fhi;  // fibers starting in the unit's window (inspector)
     float acc[RL::VPL];
@@ -158,7 +162,9 @@ cudaError_t launch_mttkrp_units(int L, const slnr_csf3& B, const float* C, const
                                 const UnitPlan& plan, cudaStream_t s) {
   if (plan.max_units <= 0 || B.nslices <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_units<W><<<grid_units(plan.max_units), 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units,
+    int ctas = grid_units(plan.max_units);  // as many as stay resident: warps take units dynamically
+    if (ctas > device_sm_count() * SLNR_MTTKRP_MIN_CTAS) ctas = device_sm_count() * SLNR_MTTKRP_MIN_CTAS;
+    k_mttkrp_units<W><<<ctas, 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units,
                                                                  plan.max_units, B.pos2, B.crd2, B.pos3,
                                                                  B.crd3, B.vals, C, D, plan.partial);
   });

@@ -17,6 +17,8 @@
 #ifndef SLNR_SDDMM_MIN_CTAS
 #define SLNR_SDDMM_MIN_CTAS 4  // resident 256-thread CTAs per SM the fused kernels are compiled for (64 registers)
 #endif
+constexpr int kRowsPerClaim = 4;  // rows a warp of the fused row kernel takes at a time
+
 #ifndef SLNR_SDDMM_U
 #define SLNR_SDDMM_U 2  // nonzeros in flight per lane group
 #endif
@@ -70,26 +72,35 @@ __device__ __forceinline__ void sddmm_spmm_range(float (&acc)[RowLanes<WM>::VPL]
 }
 
 template <int WM>
-__global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_rows(int nrows, const int32_t* __restrict__ pos,
-                                                         const int32_t* __restrict__ crd,
-                                                         const float* __restrict__ vals,
-                                                         const float* __restrict__ C,
-                                                         const float* __restrict__ D, int L,
-                                                         const float* __restrict__ E, int K,
-                                                         float* __restrict__ A) {
+__global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_rows(WsHeader* hdr, int nrows,
+                                                                              const int32_t* __restrict__ pos,
+                                                                              const int32_t* __restrict__ crd,
+                                                                              const float* __restrict__ vals,
+                                                                              const float* __restrict__ C,
+                                                                              const float* __restrict__ D, int L,
+                                                                              const float* __restrict__ E, int K,
+                                                                              float* __restrict__ A) {
   using RL = RowLanes<WM>;
   const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t r = warp; r < nrows; r += nwarps) {
-    const int p0 = pos[r], p1 = pos[r + 1];
-    if (p1 - p0 > kLightMax) continue;  // warp-uniform
-    float c[RL::VPL], acc[RL::VPL];
-    if (col < L) ldg_vec_upto<RL::VPL>(c, C + r * L + col, L - col); else zero_vec(c);
-    zero_vec(acc);
-    sddmm_spmm_range<WM>(acc, c, p0, p1, crd, vals, D, L, E, K, grp, col);
-    cross_group_sum<RL::GS>(acc);
-    if (grp == 0 && col < K) st_vec_upto(A + r * K + col, acc, K - col);
+  // warps take blocks of kRowsPerClaim rows from the header's counter until
+  // the rows run out (row lengths follow a power law: static assignment
+  // leaves warps, and the CTAs holding them, idle)
+  for (;;) {
+    int r0 = 0;
+    if (lane == 0) r0 = atomicAdd(&hdr->next_row, kRowsPerClaim);
+    r0 = __shfl_sync(0xffffffffu, r0, 0);
+    if (r0 >= nrows) break;
+    const int r1 = r0 + kRowsPerClaim < nrows ? r0 + kRowsPerClaim : nrows;
+    for (int64_t r = r0; r < r1; ++r) {
+      const int p0 = pos[r], p1 = pos[r + 1];
+      if (p1 - p0 > kLightMax) continue;  // warp-uniform
+      float c[RL::VPL], acc[RL::VPL];
+      if (col < L) ldg_vec_upto<RL::VPL>(c, C + r * L + col, L - col); else zero_vec(c);
+      zero_vec(acc);
+      sddmm_spmm_range<WM>(acc, c, p0, p1, crd, vals, D, L, E, K, grp, col);
+      cross_group_sum<RL::GS>(acc);
+      if (grp == 0 && col < K) st_vec_upto(A + r * K + col, acc, K - col);
+    }
   }
 }
 
@@ -236,11 +247,15 @@ inline int grid_rows(int64_t nwarps_needed) {
 }  // namespace
 
 cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float* D, int L,
-                                   const float* E, int K, float* A, cudaStream_t s) {
+                                   const float* E, int K, float* A, WsHeader* hdr, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
   const int WM = L > K ? L : K;
+  // as many CTAs as stay resident; hdr->next_row starts at 0 (header zeroed by the call)
+  int64_t ctas = ceil_div(ceil_div(B.nrows, kRowsPerClaim), 8);
+  const int64_t cap = (int64_t)device_sm_count() * SLNR_SDDMM_MIN_CTAS;
+  if (ctas > cap) ctas = cap;
   SLNR_WIDTH_SWITCH(WM, W, {
-    k_sddmm_spmm_rows<W><<<grid_rows(B.nrows), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A);
+    k_sddmm_spmm_rows<W><<<(unsigned)ctas, 256, 0, s>>>(hdr, B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A);
   });
   return cudaGetLastError();
 }
