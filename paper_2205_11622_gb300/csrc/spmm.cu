@@ -53,6 +53,10 @@ __global__ void __launch_bounds__(256) k_spmm_chunks(const WsHeader* __restrict_
   }
 }
 
+// Heavy rows with at most this many partials are summed by one warp when no D
+// follows (k_combine_rows); longer ones by a CTA (k_combine).
+constexpr int kWarpCombine = 16;
+
 // One CTA per heavy row: the row's partials (width W) are summed by
 // kRowLanes lanes each taking every kRowLanes-th partial, then by a fixed
 // pairwise tree, so the result does not depend on scheduling and long rows
@@ -72,6 +76,7 @@ __global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hd
   const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
   for (int h = blockIdx.x; h < n; h += gridDim.x) {
     const HeavyRow hr = heavy[h];
+    if (D == nullptr && hr.count <= kWarpCombine) continue;  // k_combine_rows writes it (block-uniform)
     float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
     if (rl < NR) {
       for (int c = rl; c < hr.count; c += NR) {
@@ -106,6 +111,45 @@ __global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hd
       }
     }
     __syncthreads();
+  }
+}
+
+// Without D, rows of at most kWarpCombine partials: a warp per heavy row
+// (grid-stride), lane l holding the columns [VPL l, VPL l + VPL); the row's
+// partials are added in their order (four loads in flight) and the sum
+// written.  Deterministic: the order is fixed.  Rows with more partials go to
+// k_combine, whose lanes split them.
+template <int W>
+__global__ void __launch_bounds__(256) k_combine_rows(const WsHeader* __restrict__ hdr,
+                                                      const HeavyRow* __restrict__ heavy, int max_heavy,
+                                                      const float* __restrict__ partial, float* __restrict__ out) {
+  using RL = RowLanes<W>;
+  const int n = min(hdr->n_heavy, max_heavy);
+  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t h = warp * RL::GPW + grp; h < n; h += nwarps * RL::GPW) {
+    const HeavyRow hr = heavy[h];
+    if (hr.count > kWarpCombine) continue;
+    float acc[RL::VPL];
+    zero_vec(acc);
+    int c = 0;
+    for (; c + 4 <= hr.count; c += 4) {
+      float x[4][RL::VPL];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) ldg_vec<RL::VPL>(x[u], partial + (int64_t)(hr.base + c + u) * W + col);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int e = 0; e < RL::VPL; ++e) acc[e] += x[u][e];
+    }
+    for (; c < hr.count; ++c) {
+      float x[RL::VPL];
+      ldg_vec<RL::VPL>(x, partial + (int64_t)(hr.base + c) * W + col);
+#pragma unroll
+      for (int e = 0; e < RL::VPL; ++e) acc[e] += x[e];
+    }
+    st_vec(out + (int64_t)hr.row * W + col, acc);
   }
 }
 
@@ -155,6 +199,14 @@ cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, 
   int grid = plan.max_heavy;
   const int cap = device_sm_count() * 8;
   if (grid > cap) grid = cap;
+  if (D == nullptr) {  // rows with few partials: a warp each; the rest below
+    SLNR_WIDTH_SWITCH(W, WC, {
+      k_combine_rows<WC><<<grid_warps(RowLanes<WC>::GPW, plan.max_heavy), 256, 0, s>>>(
+          plan.hdr, plan.heavy, plan.max_heavy, plan.partial, out);
+    });
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   SLNR_WIDTH_SWITCH(W, WC, {
     k_combine<WC><<<grid, 256, 0, s>>>(plan.hdr, plan.heavy, plan.max_heavy, plan.partial, D, L, out);
   });
