@@ -50,17 +50,48 @@ __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(WsHe
     const int flo = un.flo, fhi = un.fhi;  // fibers starting in the unit's window (inspector)
     float acc[RL::VPL];
     zero_vec(acc);
-    for (int f = flo + grp; f < fhi; f += RL::GPW) {
-      const int p0 = __ldg(pos3 + f), p1 = __ldg(pos3 + f + 1), j = __ldg(crd2 + f);
+    // The group's fibers f = flo + grp + n GPW, software-pipelined in three
+    // stages so that one round trip serves three fibers: with fiber f's rows
+    // in flight, the first nonzero (k, value) of fiber f + GPW and the record
+    // (pos3 range, j) of fiber f + 2 GPW are loaded.  Most fibers have one
+    // nonzero, whose D row then needs no further dependent load.
+    constexpr int GPW = RL::GPW;
+    auto load_rec = [&](int f, int& p0, int& p1, int& j) {
+      if (f < fhi) { p0 = __ldg(pos3 + f); p1 = __ldg(pos3 + f + 1); j = __ldg(crd2 + f); }
+      else { p0 = 0; p1 = 0; j = 0; }
+    };
+    auto load_first = [&](int p0, int p1, int& k, float& v) {
+      if (p0 < p1) { k = __ldg(crd3 + p0); v = __ldg(vals + p0); }
+      else { k = -1; v = 0.f; }
+    };
+    int f = flo + grp;
+    int p0a, p1a, ja, p0b, p1b, jb, ka;
+    float va;
+    load_rec(f, p0a, p1a, ja);
+    load_rec(f + GPW, p0b, p1b, jb);
+    load_first(p0a, p1a, ka, va);
+    for (; f < fhi; f += GPW) {
+      int kb, p0c, p1c, jc;
+      float vb;
+      load_first(p0b, p1b, kb, vb);
+      load_rec(f + 2 * GPW, p0c, p1c, jc);
       float c[RL::VPL];
-      ldg_vec<RL::VPL>(c, C + (int64_t)j * L + col);
-      // producer: T(l) = sum_k B(i,j,k) D(k,l), in registers
+      ldg_vec<RL::VPL>(c, C + (int64_t)ja * L + col);
+      // producer: T(l) = sum_k B(i,j,k) D(k,l), in registers, in nonzero order
       float t[RL::VPL];
       zero_vec(t);
-      gather_acc<RL::VPL, SLNR_MTTKRP_U>(t, crd3, vals, p0, p1, D, L, col);
+      if (ka >= 0) {
+        float x[RL::VPL];
+        ldg_vec<RL::VPL>(x, D + (int64_t)ka * L + col);
+#pragma unroll
+        for (int e = 0; e < RL::VPL; ++e) t[e] = fmaf(va, x[e], t[e]);
+        gather_acc<RL::VPL, SLNR_MTTKRP_U>(t, crd3, vals, p0a + 1, p1a, D, L, col);
+      }
       // consumer: A(i,l) += T(l) C(j,l)
 #pragma unroll
       for (int x = 0; x < RL::VPL; ++x) acc[x] = fmaf(t[x], c[x], acc[x]);
+      p0a = p0b; p1a = p1b; ja = jb; ka = kb; va = vb;
+      p0b = p0c; p1b = p1c; jb = jc;
     }
     cross_group_sum<RL::GS>(acc);
     if (grp == 0) st_vec(partial + w * L + col, acc);
@@ -100,11 +131,86 @@ __global__ void __launch_bounds__(256) k_mttkrp_stage2_units(const WsHeader* __r
   }
 }
 
-// One CTA per slice q (grid-stride): sums the slice's unit partials (strided
-// lanes, then a fixed pairwise tree) and writes A(crd1[q], :).  Rows of A
-// without a slice were zero-filled before the launch.  With E (L x M,
-// <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and A(i,:) = u(i,:).E
-// is written instead (width M): the MTTKRP result is never stored.
+// k_mttkrp_combine writes A from the unit partials: slices of more than
+// kWarpSlice units are combined by a whole CTA each, the others by one warp
+// each, in the same launch (the CTAs holding a hub slice do it first, while
+// the rest of the grid takes the small slices).
+constexpr int kWarpSlice = 16;
+
+// Warp phase: a warp per slice q (grid-stride) of at most kWarpSlice units: lane row rw
+// sums the partials rw, rw + NRW, ... in order, a fixed xor-shuffle tree adds
+// the NRW row sums (every lane ends with the same total), and A(crd1[q], :)
+// is written; with E (L x M) A(crd1[q], :) = u . E instead, lane m taking
+// outputs m, m + 32, ... with u(l) broadcast from the lane holding it.
+template <int L>
+__device__ __forceinline__ void combine_small_slices(int nslices, const int32_t* __restrict__ crd1,
+                                                     const SliceUnits* __restrict__ sus,
+                                                     const float* __restrict__ partial,
+                                                     const float* __restrict__ E, int M, float* __restrict__ A) {
+  constexpr int NC = L / 4;                  // float4 columns of a row
+  constexpr int CPL = NC > 32 ? NC / 32 : 1;  // float4 columns per lane
+  constexpr int LPR = NC / CPL;               // lanes per row
+  constexpr int NRW = 32 / LPR;               // partial rows summed at once
+  const int lane = threadIdx.x & 31, c4 = lane % LPR, rw = lane / LPR;
+  const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t q = gwarp; q < nslices; q += nwarps) {
+    const SliceUnits su = sus[q];
+    if (su.count > kWarpSlice) continue;  // warp-uniform: k_mttkrp_combine writes it
+    const int i = __ldg(crd1 + q);
+    float4 s[CPL];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) s[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int u = rw; u < su.count; u += NRW) {
+      const float4* row = reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L);
+#pragma unroll
+      for (int h = 0; h < CPL; ++h) {
+        const float4 v = __ldg(row + c4 + h * LPR);
+        s[h].x += v.x; s[h].y += v.y; s[h].z += v.z; s[h].w += v.w;
+      }
+    }
+#pragma unroll
+    for (int off = LPR; off < 32; off <<= 1)
+#pragma unroll
+      for (int h = 0; h < CPL; ++h) {
+        s[h].x += __shfl_xor_sync(0xffffffffu, s[h].x, off);
+        s[h].y += __shfl_xor_sync(0xffffffffu, s[h].y, off);
+        s[h].z += __shfl_xor_sync(0xffffffffu, s[h].z, off);
+        s[h].w += __shfl_xor_sync(0xffffffffu, s[h].w, off);
+      }
+    if (E == nullptr) {
+      if (rw == 0) {
+        float4* dst = reinterpret_cast<float4*>(A + (int64_t)i * L);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) dst[c4 + h * LPR] = s[h];
+      }
+    } else {
+      for (int m0 = 0; m0 < M; m0 += 32) {  // warp-uniform
+        const int m = m0 + lane;
+        float acc = 0.f;
+#pragma unroll
+        for (int l = 0; l < L; ++l) {
+          const int f4 = l / 4, h = f4 / LPR;
+          const float4 v = s[h];
+          const float mine = (l % 4 == 0) ? v.x : (l % 4 == 1) ? v.y : (l % 4 == 2) ? v.z : v.w;
+          const float ul = __shfl_sync(0xffffffffu, mine, f4 % LPR);
+          if (m < M) acc = fmaf(ul, __ldg(E + (int64_t)l * M + m), acc);
+        }
+        if (m < M) A[(int64_t)i * M + m] = acc;
+      }
+    }
+  }
+}
+
+// CTA phase, then the warp phase.  CTA phase: one CTA per slice q of more
+// than kWarpSlice units (grid-stride over chunks of the slices; a chunk's
+// large slices are listed first, one load per thread): sums the slice's unit
+// partials (strided lanes, each adding its partials in order with several
+// loads in flight, then a fixed pairwise tree) and writes A(crd1[q], :).
+// Rows of A without a slice were zero-filled before the launch.  With E
+// (L x M, <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and
+// A(i,:) = u(i,:).E is written instead (width M): the MTTKRP result is never
+// stored.
 template <int L>
 __global__ void __launch_bounds__(256) k_mttkrp_combine(int nslices, const int32_t* __restrict__ crd1,
                                                         const SliceUnits* __restrict__ sus,
@@ -114,39 +220,53 @@ __global__ void __launch_bounds__(256) k_mttkrp_combine(int nslices, const int32
   constexpr int NC = L / 4;
   constexpr int NR = 256 / NC;
   __shared__ float4 red[256];
+  __shared__ int big[256];
+  __shared__ int nbig;
   const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
-  for (int q = blockIdx.x; q < nslices; q += gridDim.x) {
-    const int i = __ldg(crd1 + q);
-    const SliceUnits su = sus[q];
-    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int u = rl; u < su.count; u += NR) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L) + c4);
-      s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
-    }
-    red[threadIdx.x] = s;
+  for (int64_t base = blockIdx.x; base < nslices; base += (int64_t)gridDim.x * 256) {
+    if (threadIdx.x == 0) nbig = 0;
     __syncthreads();
-    for (int half = NR / 2; half > 0; half >>= 1) {
-      if (rl < half) {
-        const float4 o = red[(rl + half) * NC + c4];
-        float4 m = red[rl * NC + c4];
-        m.x += o.x; m.y += o.y; m.z += o.z; m.w += o.w;
-        red[rl * NC + c4] = m;
+    const int64_t qt = base + (int64_t)threadIdx.x * gridDim.x;
+    if (qt < nslices && sus[qt].count > kWarpSlice) big[atomicAdd(&nbig, 1)] = (int)qt;
+    __syncthreads();
+    const int nb = nbig;
+    for (int b = 0; b < nb; ++b) {
+      const int q = big[b];
+      const int i = __ldg(crd1 + q);
+      const SliceUnits su = sus[q];
+      float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+      for (int u = rl; u < su.count; u += NR) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L) + c4);
+        s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+      }
+      red[threadIdx.x] = s;
+      __syncthreads();
+      for (int half = NR / 2; half > 0; half >>= 1) {
+        if (rl < half) {
+          const float4 o = red[(rl + half) * NC + c4];
+          float4 m = red[rl * NC + c4];
+          m.x += o.x; m.y += o.y; m.z += o.z; m.w += o.w;
+          red[rl * NC + c4] = m;
+        }
+        __syncthreads();
+      }
+      if (E == nullptr) {
+        if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
+      } else {
+        const float* uu = reinterpret_cast<const float*>(red);  // u(i,0..L)
+        for (int m = threadIdx.x; m < M; m += blockDim.x) {
+          float acc = 0.f;
+#pragma unroll 8
+          for (int l = 0; l < L; ++l) acc = fmaf(uu[l], __ldg(E + (int64_t)l * M + m), acc);
+          A[(int64_t)i * M + m] = acc;
+        }
       }
       __syncthreads();
     }
-    if (E == nullptr) {
-      if (rl == 0) reinterpret_cast<float4*>(A + (int64_t)i * L)[c4] = red[c4];
-    } else {
-      const float* uu = reinterpret_cast<const float*>(red);  // u(i,0..L)
-      for (int m = threadIdx.x; m < M; m += blockDim.x) {
-        float acc = 0.f;
-#pragma unroll 8
-        for (int l = 0; l < L; ++l) acc = fmaf(uu[l], __ldg(E + (int64_t)l * M + m), acc);
-        A[(int64_t)i * M + m] = acc;
-      }
-    }
-    __syncthreads();
+    __syncthreads();  // every thread has read nbig before the next chunk resets it
   }
+  combine_small_slices<L>(nslices, crd1, sus, partial, E, M, A);
 }
 
 inline int grid_units(int64_t max_units) {
@@ -187,11 +307,12 @@ cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& pla
   // rows of A without a slice are zero; the kernel writes the others
   cudaError_t e = cudaMemsetAsync(A, 0, sizeof(float) * (size_t)B.dim[0] * (size_t)(E != nullptr ? M : L), s);
   if (e != cudaSuccess || B.nslices <= 0) return e;
-  int grid = B.nslices;
-  const int cap = device_sm_count() * 8;
-  if (grid > cap) grid = cap;
+  // a warp per slice in the warp phase (8 per CTA); grid-stride beyond
+  int64_t grid = ceil_div(B.nslices, 8);
+  if (grid > (int64_t)device_sm_count() * 32) grid = (int64_t)device_sm_count() * 32;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_combine<W><<<grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial, E, M, A);
+    k_mttkrp_combine<W><<<(unsigned)grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial, E, M,
+                                                       A);
   });
   return cudaGetLastError();
 }

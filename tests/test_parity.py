@@ -79,6 +79,15 @@ def test_mttkrp_widths(slnr, orc, L, variant):
     check(slnr, orc, w, variant)
 
 
+@pytest.mark.parametrize("L", [4, 32, 256])
+@pytest.mark.parametrize("variant", ["fused", "unfused"])
+def test_mttkrp_hub_slice(slnr, orc, L, variant):
+    # Zipf(1.6) over 40 slices: one slice of more than 16 units (512 nonzeros
+    # each) is combined by a CTA, the other 39 by a warp each
+    w = wl.mttkrp_zipf(0x51A5, (40, 200, 400), 40000, 1.6, L)
+    check(slnr, orc, w, variant)
+
+
 @pytest.mark.parametrize("L,M", [(4, 16), (16, 4), (16, 16), (16, 64), (32, 16), (32, 64), (64, 64), (128, 32),
                                  (128, 256), (256, 128)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])

@@ -69,6 +69,15 @@ def test_mttkrp_gemm_widths(slnr, orc, L, M, variant):
     check(slnr, orc, w, variant, True)
 
 
+@pytest.mark.parametrize("L,M", [(4, 8), (32, 64), (256, 16)])
+@pytest.mark.parametrize("variant", ["fused", "unfused"])
+def test_mttkrp_gemm_hub_slice(slnr, orc, L, M, variant):
+    # one slice of more than 16 units (combined by a CTA), 39 small ones (a warp each)
+    w = wl.mttkrp_gemm_zipf(0x51A5, (40, 200, 400), 40000, 1.6, L, M)
+    check(slnr, orc, w, variant, False)
+    check(slnr, orc, w, variant, True)
+
+
 @pytest.mark.parametrize("J,L", [(4, 8), (16, 256), (32, 32), (64, 128), (128, 64), (128, 128), (256, 64)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_spmmh_gemm_widths(slnr, orc, J, L, variant):
