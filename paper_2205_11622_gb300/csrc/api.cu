@@ -81,13 +81,14 @@ struct Layout {
     o_partial = take(sizeof(float) * (size_t)max_chunks * (size_t)width);
   }
   // MTTKRP units
-  size_t o_su = 0, o_units = 0, o_upartial = 0;
+  size_t o_su = 0, o_units = 0, o_upartial = 0, o_uparts = 0;
   int max_units = 0;
   void units(int64_t nslices, int64_t nnz, int width) {
     max_units = (int)(nnz / kUnitNnz + nslices + 1);
     o_su = take(sizeof(SliceUnits) * (size_t)nslices);
     o_units = take(sizeof(Unit) * (size_t)max_units);
     o_upartial = take(sizeof(float) * (size_t)max_units * (size_t)width);
+    o_uparts = take(sizeof(float) * (size_t)max_units * (size_t)width);
   }
   // row segments of the tensor-core path (partials are A rows of the output width)
   size_t o_counts = 0, o_segs = 0;
@@ -133,7 +134,7 @@ SplitPlan combine_plan(const SegPlan& g) {
 UnitPlan unit_plan(char* ws, const Layout& l) {
   return UnitPlan{reinterpret_cast<WsHeader*>(ws), reinterpret_cast<SliceUnits*>(ws + l.o_su),
                   reinterpret_cast<Unit*>(ws + l.o_units), reinterpret_cast<float*>(ws + l.o_upartial),
-                  l.max_units};
+                  l.max_units, reinterpret_cast<float*>(ws + l.o_uparts)};
 }
 
 // ---------------------------------------------------------------------------

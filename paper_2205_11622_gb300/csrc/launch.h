@@ -39,6 +39,7 @@ struct UnitPlan {
   Unit* units;              // [max_units]
   float* partial;           // max_units x L
   int max_units;
+  float* part_sums;         // max_units x L: sums of runs of kPartUnits unit partials of large slices
 };
 
 // Workspace pieces of the tensor-core path: row segments of at most

@@ -202,11 +202,79 @@ __device__ __forceinline__ void combine_small_slices(int nslices, const int32_t*
   }
 }
 
+// A slice of more than kWarpSlice units is summed in two levels: runs of
+// kPartUnits consecutive unit partials first (k_mttkrp_parts, a warp per run,
+// so a hub slice of thousands of units spreads over the GPU), then its part
+// sums by one CTA (k_mttkrp_combine).  Both levels add in a fixed order.
+constexpr int kPartUnits = 64;
+
+// A warp per run: each lane checks one unit, the run leaders (unit u of a
+// large slice with u a multiple of kPartUnits) are taken in turn by the whole
+// warp.  Lane row rw adds the run's partials rw, rw + NRW, ... in order, a
+// fixed xor-shuffle tree adds the row sums, and the sum is written to
+// part_sums row base + u / kPartUnits (inside the slice's own unit range).
+template <int L>
+__global__ void __launch_bounds__(256) k_mttkrp_parts(const WsHeader* __restrict__ hdr,
+                                                      const Unit* __restrict__ units,
+                                                      const SliceUnits* __restrict__ sus, int max_units,
+                                                      const float* __restrict__ partial,
+                                                      float* __restrict__ part_sums) {
+  constexpr int NC = L / 4;
+  constexpr int CPL = NC > 32 ? NC / 32 : 1;
+  constexpr int LPR = NC / CPL;
+  constexpr int NRW = 32 / LPR;
+  const int n = min(hdr->n_units, max_units);
+  const int lane = threadIdx.x & 31, c4 = lane % LPR, rw = lane / LPR;
+  const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t w0 = gwarp * 32; w0 < n; w0 += nwarps * 32) {
+    bool lead = false;
+    if (w0 + lane < n) {
+      const Unit un = units[w0 + lane];
+      lead = un.u % kPartUnits == 0 && sus[un.slice].count > kWarpSlice;
+    }
+    unsigned m = __ballot_sync(0xffffffffu, lead);
+    while (m != 0) {  // warp-uniform
+      const int b = __ffs(m) - 1;
+      m &= m - 1;
+      const Unit un = units[w0 + b];
+      const SliceUnits su = sus[un.slice];
+      const int u1 = min(un.u + kPartUnits, su.count);
+      float4 s[CPL];
+#pragma unroll
+      for (int h = 0; h < CPL; ++h) s[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+      for (int u = un.u + rw; u < u1; u += NRW) {
+        const float4* row = reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+          const float4 v = __ldg(row + c4 + h * LPR);
+          s[h].x += v.x; s[h].y += v.y; s[h].z += v.z; s[h].w += v.w;
+        }
+      }
+#pragma unroll
+      for (int off = LPR; off < 32; off <<= 1)
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+          s[h].x += __shfl_xor_sync(0xffffffffu, s[h].x, off);
+          s[h].y += __shfl_xor_sync(0xffffffffu, s[h].y, off);
+          s[h].z += __shfl_xor_sync(0xffffffffu, s[h].z, off);
+          s[h].w += __shfl_xor_sync(0xffffffffu, s[h].w, off);
+        }
+      if (rw == 0) {
+        float4* dst = reinterpret_cast<float4*>(part_sums + (int64_t)(su.base + un.u / kPartUnits) * L);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) dst[c4 + h * LPR] = s[h];
+      }
+    }
+  }
+}
+
 // CTA phase, then the warp phase.  CTA phase: one CTA per slice q of more
 // than kWarpSlice units (grid-stride over chunks of the slices; a chunk's
-// large slices are listed first, one load per thread): sums the slice's unit
-// partials (strided lanes, each adding its partials in order with several
-// loads in flight, then a fixed pairwise tree) and writes A(crd1[q], :).
+// large slices are listed first, one load per thread): sums the slice's part
+// sums (strided lanes, each adding in order, then a fixed pairwise tree) and
+// writes A(crd1[q], :).
 // Rows of A without a slice were zero-filled before the launch.  With E
 // (L x M, <MTTKRP,GEMM>) the row u(i,:) stays in shared memory and
 // A(i,:) = u(i,:).E is written instead (width M): the MTTKRP result is never
@@ -215,6 +283,7 @@ template <int L>
 __global__ void __launch_bounds__(256) k_mttkrp_combine(int nslices, const int32_t* __restrict__ crd1,
                                                         const SliceUnits* __restrict__ sus,
                                                         const float* __restrict__ partial,
+                                                        const float* __restrict__ part_sums,
                                                         const float* __restrict__ E, int M,
                                                         float* __restrict__ A) {
   constexpr int NC = L / 4;
@@ -234,10 +303,11 @@ __global__ void __launch_bounds__(256) k_mttkrp_combine(int nslices, const int32
       const int q = big[b];
       const int i = __ldg(crd1 + q);
       const SliceUnits su = sus[q];
+      const int np = (su.count + kPartUnits - 1) / kPartUnits;  // its part sums (k_mttkrp_parts)
       float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-      for (int u = rl; u < su.count; u += NR) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(partial + (int64_t)(su.base + u) * L) + c4);
+#pragma unroll 4
+      for (int u = rl; u < np; u += NR) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(part_sums + (int64_t)(su.base + u) * L) + c4);
         s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
       }
       red[threadIdx.x] = s;
@@ -311,8 +381,12 @@ cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& pla
   int64_t grid = ceil_div(B.nslices, 8);
   if (grid > (int64_t)device_sm_count() * 32) grid = (int64_t)device_sm_count() * 32;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_combine<W><<<(unsigned)grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial, E, M,
-                                                       A);
+    int64_t pgrid = ceil_div(plan.max_units, 32 * 8);  // a warp per 32 units
+    if (pgrid > (int64_t)device_sm_count() * 32) pgrid = (int64_t)device_sm_count() * 32;
+    k_mttkrp_parts<W><<<(unsigned)pgrid, 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units, plan.max_units,
+                                                      plan.partial, plan.part_sums);
+    k_mttkrp_combine<W><<<(unsigned)grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial,
+                                                       plan.part_sums, E, M, A);
   });
   return cudaGetLastError();
 }

@@ -82,9 +82,10 @@ def test_mttkrp_widths(slnr, orc, L, variant):
 @pytest.mark.parametrize("L", [4, 32, 256])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_mttkrp_hub_slice(slnr, orc, L, variant):
-    # Zipf(1.6) over 40 slices: one slice of more than 16 units (512 nonzeros
-    # each) is combined by a CTA, the other 39 by a warp each
-    w = wl.mttkrp_zipf(0x51A5, (40, 200, 400), 40000, 1.6, L)
+    # Zipf(1.8) over 40 slices: 3 slices of more than 16 units (512 nonzeros
+    # each; the largest has 162, i.e. 3 runs of at most 64 units, the last one
+    # ragged) are summed in two levels, the other 37 by a warp each
+    w = wl.mttkrp_zipf(0x51A5, (40, 400, 500), 150000, 1.8, L)
     check(slnr, orc, w, variant)
 
 

@@ -72,8 +72,9 @@ def test_mttkrp_gemm_widths(slnr, orc, L, M, variant):
 @pytest.mark.parametrize("L,M", [(4, 8), (32, 64), (256, 16)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_mttkrp_gemm_hub_slice(slnr, orc, L, M, variant):
-    # one slice of more than 16 units (combined by a CTA), 39 small ones (a warp each)
-    w = wl.mttkrp_gemm_zipf(0x51A5, (40, 200, 400), 40000, 1.6, L, M)
+    # 3 slices of more than 16 units (two-level sums, the largest in 3 runs of
+    # at most 64 units), 37 small ones (a warp each)
+    w = wl.mttkrp_gemm_zipf(0x51A5, (40, 400, 500), 150000, 1.8, L, M)
     check(slnr, orc, w, variant, False)
     check(slnr, orc, w, variant, True)
 
