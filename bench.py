@@ -593,6 +593,9 @@ def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_fl
         for t in (o if isinstance(o, tuple) else (o,)):
             dev_out[i].append(t)
             host_out[i].append(torch.empty(t.shape, dtype=t.dtype, pin_memory=True))
+    # the device-resident path's outputs for the same inputs: the read-back
+    # outputs must equal them bit for bit (every kernel sums in a fixed order)
+    expect = [[t.cpu() for t in dev_out[i]] for i in range(n)]
     h2d = sum(t.numel() * t.element_size() for hs in host_in for t in hs)
     d2h = sum(t.numel() * t.element_size() for hs in host_out for t in hs)
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
@@ -637,13 +640,16 @@ def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_fl
     b.record(stream)
     b.synchronize()
     ms = a.elapsed_time(b) / steps
+    torch.cuda.synchronize()
+    differ = sum(int(not torch.equal(h, e)) for i in range(n) for h, e in zip(host_out[i], expect[i]))
     if pg is not None:
         t = torch.tensor([ms], dtype=torch.float64, device=dev)
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
         ms = float(t.item())
     return {"value": round(world * total_flops / (ms / 1e3) / 1e9, 2), "unit": "GFLOP/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 3),
-            "link_gbs": round((h2d + d2h) / (ms / 1e3) / 1e9, 1)}
+            "link_gbs": round((h2d + d2h) / (ms / 1e3) / 1e9, 1),
+            "outputs_read_back": sum(len(x) for x in expect), "outputs_differing_from_device_path": differ}
 
 
 if __name__ == "__main__":
