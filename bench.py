@@ -83,8 +83,8 @@ def row_flops(w) -> np.ndarray:
         L = d["L"]
         f = np.zeros(w.B.dims[0], np.int64)
         if w.B.nslices:
-            fib_nnz = np.diff(w.B.pos3).astype(np.int64)
-            nnz_s = np.add.reduceat(fib_nnz, w.B.pos2[:-1]) if w.B.nfibers else np.zeros(w.B.nslices, np.int64)
+            pos3 = w.B.pos3.astype(np.int64)
+            nnz_s = np.diff(pos3[w.B.pos2])           # nonzeros per slice (0 for a slice without fibers)
             nfib_s = np.diff(w.B.pos2).astype(np.int64)
             f[w.B.crd1] = 2 * nnz_s * L + 2 * nfib_s * L
             if w.op == "mttkrp_gemm":
