@@ -30,7 +30,9 @@
  *    index arrays on the device, waits for that check on the stream, and
  *    returns SLNR_ERR_INDEX (enqueuing nothing else) if they are malformed.
  *    With validate == 0 the indices are trusted; malformed indices are then
- *    undefined behaviour.
+ *    undefined behaviour.  In validate mode the call also waits for its
+ *    kernels at the end and returns SLNR_ERR_TIMEOUT if a bounded device-side
+ *    wait gave up (see slnr_set_wait_limit).
  *  - opts->workspace must hold at least the number of bytes that the
  *    matching slnr_*_workspace query reports for the same arguments, and be
  *    256-byte aligned.  Its contents need no initialisation; calls that share
@@ -231,6 +233,19 @@ slnr_status slnr_timing_enable(int32_t on);
 int32_t slnr_timing_count(void);
 /* Name of launch i of the last call and its device time in milliseconds. */
 slnr_status slnr_timing_get(int32_t i, const char **name, float *ms);
+
+/* ---- bounded device-side waits ------------------------------------------
+ * Every spin of the tensor-core kernels (on an mbarrier, a shared counter or
+ * the tile-index ring) gives up after a limit of SM clock cycles, sets the
+ * timeout bit of the workspace flag word and winds the CTA down (MMAs
+ * already issued are drained, with the default limit, before the tensor
+ * memory is freed).  A call with opts->validate != 0 waits for its launches
+ * and returns SLNR_ERR_TIMEOUT when that bit is set.  This sets the limit
+ * that the calling thread's later calls give those waits: cycles = 0
+ * restores the default (4e9 cycles, about 2 s at 2 GHz).  Meant for testing
+ * the timeout path; a limit shorter than the work makes correct calls fail.
+ * Returns SLNR_ERR_SHAPE for cycles < 0. */
+slnr_status slnr_set_wait_limit(int64_t cycles);
 
 /* ---- diagnostics ------------------------------------------------------- */
 const char *slnr_status_string(slnr_status status);

@@ -71,6 +71,7 @@ SIGNATURES = {
     "slnr_mttkrp_gemm": ([_CSF, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_spmmh_gemm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_sddmm_spmm_noalloc": ([_CSR, _P, _P, _I32, _P, _I32, _P, _P], ctypes.c_int),
+    "slnr_set_wait_limit": ([ctypes.c_int64], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
     "slnr_timing_get": ([_I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),

@@ -11,6 +11,7 @@ using namespace slnr;
 namespace {
 
 thread_local char g_last_error[512] = "";
+thread_local long long g_wait_limit = 0;  // 0: kWaitCycles
 
 slnr_status fail(slnr_status st, const char* fmt, ...) {
   va_list ap;
@@ -103,7 +104,7 @@ struct Layout {
     max_heavy = (int)mh;
     max_chunks = (int)mc;
     max_segs = (int)(nrows + mc);
-    o_counts = take(sizeof(int) * 3 * (size_t)seg_scan_blocks(nrows));
+    o_counts = take(sizeof(int) * kSegCounters * (size_t)seg_scan_blocks(nrows));
     o_segs = take(sizeof(int4) * (size_t)max_segs);
     o_heavy = take(sizeof(HeavyRow) * (size_t)mh);
     o_partial = take(sizeof(float) * (size_t)mc * (size_t)width);
@@ -226,6 +227,22 @@ slnr_status begin(char* ws, cudaStream_t s, bool validate, Launch launch_validat
   return SLNR_OK;
 }
 
+// End of a call.  In validate mode the call waits for its launches and reads
+// the device flag word: a bounded wait that gave up returns SLNR_ERR_TIMEOUT,
+// an inspector bound exceeded (positions inconsistent with nnz) returns
+// SLNR_ERR_INDEX.  Otherwise the launches stay asynchronous.
+slnr_status finish(char* ws, cudaStream_t s, bool validate) {
+  timing_end(s);
+  if (!validate) return SLNR_OK;
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(ws);
+  int flag = 0;
+  SLNR_CUDA(cudaMemcpyAsync(&flag, &hdr->error, sizeof(int), cudaMemcpyDeviceToHost, s));
+  SLNR_CUDA(cudaStreamSynchronize(s));
+  if (flag & kErrTimeout) return fail(SLNR_ERR_TIMEOUT, "a bounded device-side wait gave up (flags 0x%x)", flag);
+  if (flag != 0) return fail(SLNR_ERR_INDEX, "the inspector found more work than the sizes allow (flags 0x%x)", flag);
+  return SLNR_OK;
+}
+
 // ---------------------------------------------------------------------------
 // layouts per operation
 
@@ -302,6 +319,8 @@ CsrView fiber_view(const slnr_csf3* B) {
 
 void slnr::set_last_error(const char* msg) { snprintf(g_last_error, sizeof(g_last_error), "%s", msg); }
 
+long long slnr::wait_limit_cycles() { return g_wait_limit > 0 ? g_wait_limit : kWaitCycles; }
+
 // ===========================================================================
 
 extern "C" {
@@ -322,7 +341,13 @@ const char* slnr_status_string(slnr_status s) {
 
 const char* slnr_last_error(void) { return g_last_error; }
 
-const char* slnr_version(void) { return "slnr 0.1.0 (sm_103a)"; }
+const char* slnr_version(void) { return "slnr 0.2.0 (sm_103a)"; }
+
+slnr_status slnr_set_wait_limit(int64_t cycles) {
+  if (cycles < 0) return fail(SLNR_ERR_SHAPE, "wait limit must be >= 0");
+  g_wait_limit = cycles;
+  return SLNR_OK;
+}
 
 slnr_status slnr_timing_enable(int32_t on) {
   if (on && !g_timing.created) {
@@ -464,8 +489,7 @@ slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const f
         SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, K, L, T, D, A, 0, s));
     }
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_sddmm_spmm(const slnr_csr* B, const float* C, const float* D, int32_t L, const float* E,
@@ -504,8 +528,7 @@ slnr_status slnr_sddmm_spmm(const slnr_csr* B, const float* C, const float* D, i
     SLNR_LAUNCH("spmm_rows", launch_spmm_rows(K, vy, E, A, s));
     SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, A, s));
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_mttkrp(const slnr_csf3* B, const float* C, const float* D, int32_t L, float* A,
@@ -540,8 +563,7 @@ slnr_status slnr_mttkrp(const slnr_csf3* B, const float* C, const float* D, int3
     SLNR_LAUNCH("mttkrp_stage2_units", launch_mttkrp_stage2_units(L, *B, T, C, up, s));
   }
   SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, nullptr, 0, A, s));
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const float* D, int32_t M,
@@ -598,8 +620,7 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
         SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nfibers, L, M, T, D, A_vals, 0, s));
     }
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float* D, int32_t K, const float* F,
@@ -646,8 +667,7 @@ slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float*
     else
       SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, L, M, T, W, A, 0, s));
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_mttkrp_gemm(const slnr_csf3* B, const float* C, const float* D, int32_t L, const float* E,
@@ -690,8 +710,7 @@ slnr_status slnr_mttkrp_gemm(const slnr_csf3* B, const float* C, const float* D,
     else
       SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->dim[0], L, M, U, E, A, 0, s));
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 slnr_status slnr_spmmh_gemm(const slnr_csr* B, const float* C, const float* D, int32_t J, const float* E,
@@ -739,8 +758,7 @@ slnr_status slnr_spmmh_gemm(const slnr_csr* B, const float* C, const float* D, i
         SLNR_LAUNCH("dense_gemm", launch_dense_gemm(B->nrows, J, L, T, E, A, 0, s));
     }
   }
-  timing_end(s);
-  return SLNR_OK;
+  return finish(ws, s, opts->validate != 0);
 }
 
 }  // extern "C"

@@ -22,8 +22,13 @@ constexpr int kChunk = 256;
 // MTTKRP: a slice is cut into units of fibers that start within one window
 // of kUnitNnz nonzeros.
 constexpr int kUnitNnz = 512;
-// Tensor-core path: rows are cut into segments of at most kSegChunk nonzeros.
+// Tensor-core path: rows are cut into segments of at most kSegChunk nonzeros,
+// listed by length class (kSegClasses classes: (64,128], (32,64], ..., 2, 1,
+// empty); the inspector keeps kSegCounters counters per block of rows (one
+// per class, heavy rows, chunks of heavy rows).
 constexpr int kSegChunk = 128;
+constexpr int kSegClasses = 9;
+constexpr int kSegCounters = kSegClasses + 2;
 
 struct WsHeader {        // first 256 bytes of every workspace
   int n_heavy;           // heavy rows found by the inspector

@@ -46,7 +46,7 @@ struct UnitPlan {
 // kSegChunk nonzeros (tc_gemm.cu).
 struct SegPlan {
   WsHeader* hdr;
-  int* block_counts;  // 3 ints per inspector block
+  int* block_counts;  // kSegCounters ints per inspector block
   int4* segs;         // {row, p0, p1, partial slot or -1}
   HeavyRow* heavy;
   float* partial;     // max_chunks x L partial A rows
@@ -59,6 +59,13 @@ int device_sm_count();
 
 // Sets the calling thread's slnr_last_error() text (api.cu).
 void set_last_error(const char* msg);
+
+// Default limit, in SM clock cycles, of every bounded device-side wait
+// (about 2 s at 2 GHz).
+constexpr long long kWaitCycles = 4000000000LL;
+// The limit the calling thread's launches give their bounded waits
+// (kWaitCycles unless slnr_set_wait_limit changed it; api.cu).
+long long wait_limit_cycles();
 
 // inspect.cu
 cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_t s);

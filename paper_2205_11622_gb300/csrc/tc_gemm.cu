@@ -27,21 +27,38 @@ namespace slnr {
 
 namespace {
 
-constexpr int kTcThreads = 1024;
+#ifndef SLNR_TC_WARPS
+#define SLNR_TC_WARPS 32  // warps of the tile kernel's CTA: producers, then one MMA warp, then four epilogue warps
+#endif
+constexpr int kTcWarps = SLNR_TC_WARPS;
+constexpr int kTcThreads = 32 * kTcWarps;
+static_assert(kTcWarps % 4 == 0 && kTcWarps >= 8, "the four epilogue warps are a whole warpgroup");
 constexpr int kTcRows = 128;  // MMA M
 constexpr int kScanRows = 2048;
 constexpr int kScanThreads = 256;
 constexpr int kRowsPerThread = kScanRows / kScanThreads;
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 __device__ __forceinline__ int segs_of(int n) { return n <= kSegChunk ? 1 : (n + kSegChunk - 1) / kSegChunk; }
 
-// Inclusive block scan of 3 ints (kScanThreads threads); returns block totals in tot.
-__device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3]) {
-  __shared__ int wsum[kScanThreads / 32][3];
+// Segments are listed by length class, longest first, so that the items a
+// lane group takes together have similar lengths and one batch shape fits
+// them all (a short segment would otherwise pay for a whole predicated batch
+// of row loads).  Class of a segment of n nonzeros: n in (64,128] -> 0,
+// (32,64] -> 1, ..., 2 -> 6, 1 -> 7, empty -> 8.  Long segments first also
+// keeps the costly item tiles away from the end of the kernel.
+__device__ __forceinline__ int seg_class(int n) {
+  const int c = n <= 1 ? 0 : 32 - __clz(n - 1);  // ceil(log2(n)) for n >= 1
+  return n == 0 ? kSegClasses - 1 : kSegClasses - 2 - c;
+}
+
+// Inclusive block scan of N ints (kScanThreads threads); returns the block
+// totals in tot.
+template <int N>
+__device__ __forceinline__ void block_scan(int (&v)[N], int (&tot)[N]) {
+  __shared__ int wsum[kScanThreads / 32][N];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-  for (int q = 0; q < 3; ++q)
+  for (int q = 0; q < N; ++q)
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, v[q], o);
@@ -49,10 +66,10 @@ __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3]) {
     }
   if (lane == 31)
 #pragma unroll
-    for (int q = 0; q < 3; ++q) wsum[warp][q] = v[q];
+    for (int q = 0; q < N; ++q) wsum[warp][q] = v[q];
   __syncthreads();
 #pragma unroll
-  for (int q = 0; q < 3; ++q) {
+  for (int q = 0; q < N; ++q) {
     int before = 0, all = 0;
     for (int w = 0; w < kScanThreads / 32; ++w) {
       if (w < warp) before += wsum[w][q];
@@ -64,95 +81,126 @@ __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3]) {
   __syncthreads();
 }
 
-// Pass 1: per block of kScanRows rows, the number of segments, heavy rows and
-// heavy-row chunks.
+// Adds one row of n nonzeros to the counters: segments per class
+// (kSegClasses of them), then heavy rows, then chunks of heavy rows.
+__device__ __forceinline__ void count_row(int n, int (&v)[kSegCounters]) {
+  const int ns = segs_of(n);
+  const int q = seg_class(ns == 1 ? n : n - (ns - 1) * kSegChunk);  // the row's (last) segment
+#pragma unroll
+  for (int k = 0; k < kSegClasses; ++k) v[k] += (k == q) + (k == 0 ? ns - 1 : 0);  // full chunks: class 0
+  v[kSegClasses] += ns > 1;
+  v[kSegClasses + 1] += ns > 1 ? ns : 0;
+}
+
+// Pass 1: the counters of each block of kScanRows rows.
 __global__ void __launch_bounds__(kScanThreads) k_seg_count(int nrows, const int32_t* __restrict__ pos,
                                                             int* __restrict__ counts) {
   const int64_t r0 = (int64_t)blockIdx.x * kScanRows + (int64_t)threadIdx.x * kRowsPerThread;
-  int v[3] = {0, 0, 0};
+  int v[kSegCounters] = {};
   for (int i = 0; i < kRowsPerThread; ++i) {
     const int64_t r = r0 + i;
-    if (r < nrows) {
-      const int ns = segs_of(pos[r + 1] - pos[r]);
-      v[0] += ns;
-      if (ns > 1) {
-        v[1] += 1;
-        v[2] += ns;
-      }
-    }
+    if (r < nrows) count_row(pos[r + 1] - pos[r], v);
   }
-  int tot[3];
-  block_scan3(v, tot);
-  if (threadIdx.x == 0) {
-    counts[3 * blockIdx.x + 0] = tot[0];
-    counts[3 * blockIdx.x + 1] = tot[1];
-    counts[3 * blockIdx.x + 2] = tot[2];
-  }
+  int tot[kSegCounters];
+  block_scan<kSegCounters>(v, tot);
+  if (threadIdx.x < kSegCounters) counts[kSegCounters * blockIdx.x + threadIdx.x] = tot[threadIdx.x];
 }
 
-// Pass 2: each block adds up the counts of the blocks before it, scans its
-// rows and writes their segments (in row order), heavy-row records and chunk
-// slots.  The last block publishes the totals in the workspace header.
+// Pass 2: each block adds up the counters of all blocks (the class sizes) and
+// of the blocks before it, scans its rows and writes their segments into
+// their classes' ranges (row order within a class), the heavy-row records
+// and the chunk slots (row order).  No atomic decides a position, so the
+// lists are the same on every run.  Block 0 publishes the totals in the
+// workspace header.
 __global__ void __launch_bounds__(kScanThreads) k_seg_write(int nrows, const int32_t* __restrict__ pos,
                                                             const int* __restrict__ counts, int nblocks,
                                                             WsHeader* hdr, int4* __restrict__ segs,
                                                             HeavyRow* __restrict__ heavy, int max_segs,
                                                             int max_heavy, int max_chunks) {
-  __shared__ int base[3];
-  if (threadIdx.x < 3) base[threadIdx.x] = 0;
+  __shared__ int pre_s[kSegCounters], all_s[kSegCounters];
+  if (threadIdx.x < kSegCounters) pre_s[threadIdx.x] = all_s[threadIdx.x] = 0;
   __syncthreads();
-  int pre[3] = {0, 0, 0};
-  for (int b = threadIdx.x; b < (int)blockIdx.x; b += blockDim.x) {
-    pre[0] += counts[3 * b + 0];
-    pre[1] += counts[3 * b + 1];
-    pre[2] += counts[3 * b + 2];
-  }
+  {
+    int pre[kSegCounters] = {}, all[kSegCounters] = {};
+    for (int b = threadIdx.x; b < nblocks; b += blockDim.x)
 #pragma unroll
-  for (int q = 0; q < 3; ++q) {
-    int x = pre[q];
+      for (int q = 0; q < kSegCounters; ++q) {
+        const int x = counts[kSegCounters * b + q];
+        all[q] += x;
+        if (b < (int)blockIdx.x) pre[q] += x;
+      }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    if ((threadIdx.x & 31) == 0 && x != 0) atomicAdd(&base[q], x);
-  }
-  __syncthreads();
-  const int64_t r0 = (int64_t)blockIdx.x * kScanRows + (int64_t)threadIdx.x * kRowsPerThread;
-  int v[3] = {0, 0, 0};
-  for (int i = 0; i < kRowsPerThread; ++i) {
-    const int64_t r = r0 + i;
-    if (r < nrows) {
-      const int ns = segs_of(pos[r + 1] - pos[r]);
-      v[0] += ns;
-      if (ns > 1) {
-        v[1] += 1;
-        v[2] += ns;
+    for (int q = 0; q < kSegCounters; ++q) {
+      int x = pre[q], y = all[q];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        x += __shfl_xor_sync(0xffffffffu, x, o);
+        y += __shfl_xor_sync(0xffffffffu, y, o);
+      }
+      if ((threadIdx.x & 31) == 0) {
+        if (x != 0) atomicAdd(&pre_s[q], x);
+        if (y != 0) atomicAdd(&all_s[q], y);
       }
     }
   }
-  const int mine[3] = {v[0], v[1], v[2]};
-  int tot[3];
-  block_scan3(v, tot);
-  int so = base[0] + v[0] - mine[0], ho = base[1] + v[1] - mine[1], co = base[2] + v[2] - mine[2];
+  __syncthreads();
+  const int64_t r0 = (int64_t)blockIdx.x * kScanRows + (int64_t)threadIdx.x * kRowsPerThread;
+  int v[kSegCounters] = {};
+  for (int i = 0; i < kRowsPerThread; ++i) {
+    const int64_t r = r0 + i;
+    if (r < nrows) count_row(pos[r + 1] - pos[r], v);
+  }
+  int at[kSegCounters];
+#pragma unroll
+  for (int q = 0; q < kSegCounters; ++q) at[q] = v[q];
+  int tot[kSegCounters];
+  block_scan<kSegCounters>(v, tot);
+  // at[q]: this thread's first position of counter q (classes: within the
+  // whole list, after the classes that come before it)
+  int cls_start = 0;
+#pragma unroll
+  for (int q = 0; q < kSegCounters; ++q) {
+    at[q] = pre_s[q] + v[q] - at[q] + (q < kSegClasses ? cls_start : 0);
+    if (q < kSegClasses) cls_start += all_s[q];
+  }
+  auto put = [&](int n, int4 rec) {
+    const int q = seg_class(n);
+#pragma unroll
+    for (int k = 0; k < kSegClasses; ++k)
+      if (k == q) {
+        if (at[k] < max_segs) segs[at[k]] = rec;
+        ++at[k];
+      }
+  };
   for (int i = 0; i < kRowsPerThread; ++i) {
     const int64_t r = r0 + i;
     if (r >= nrows) break;
     const int p0 = pos[r], p1 = pos[r + 1];
     const int ns = segs_of(p1 - p0);
     if (ns == 1) {
-      if (so < max_segs) segs[so] = make_int4((int)r, p0, p1, -1);
-      ++so;
+      put(p1 - p0, make_int4((int)r, p0, p1, -1));
     } else {
-      if (ho < max_heavy && co + ns <= max_chunks) heavy[ho] = HeavyRow{(int)r, co, ns, 0};
-      ++ho;
-      for (int c = 0; c < ns; ++c) {
-        const int a = p0 + c * kSegChunk;
-        if (so < max_segs && co < max_chunks) segs[so] = make_int4((int)r, a, min(p1, a + kSegChunk), co);
-        ++so;
-        ++co;
-      }
+      const int ho = at[kSegClasses], co = at[kSegClasses + 1];
+      const bool fits = ho < max_heavy && co + ns <= max_chunks;
+      if (fits) heavy[ho] = HeavyRow{(int)r, co, ns, 0};
+      at[kSegClasses] += 1;
+      at[kSegClasses + 1] += ns;
+      // the ns - 1 full chunks are consecutive in the first class, then the
+      // last chunk goes to its own class
+      const int f0 = at[0];
+      at[0] += ns - 1;
+      for (int c = 0; c < ns - 1; ++c)
+        if (f0 + c < max_segs)
+          segs[f0 + c] = make_int4((int)r, p0 + c * kSegChunk, p0 + (c + 1) * kSegChunk, fits ? co + c : -1);
+      const int a = p0 + (ns - 1) * kSegChunk;
+      put(p1 - a, make_int4((int)r, a, p1, fits ? co + ns - 1 : -1));
     }
   }
-  if (blockIdx.x == nblocks - 1 && threadIdx.x == 0) {
-    const int ns = base[0] + tot[0], nh = base[1] + tot[1], nc = base[2] + tot[2];
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    int ns = 0;
+#pragma unroll
+    for (int q = 0; q < kSegClasses; ++q) ns += all_s[q];
+    const int nh = all_s[kSegClasses], nc = all_s[kSegClasses + 1];
     hdr->n_segs = ns;
     hdr->n_heavy = nh;
     hdr->n_chunks = nc;
@@ -160,12 +208,13 @@ __global__ void __launch_bounds__(kScanThreads) k_seg_write(int nrows, const int
   }
 }
 
-// Waits until *count >= target (a monotonic shared-memory counter); false on timeout.
-__device__ __forceinline__ bool count_wait_timeout(const int* count, int target) {
+// Waits until *count >= target (a monotonic shared-memory counter); false
+// after `limit` clock cycles.
+__device__ __forceinline__ bool count_wait_timeout(const int* count, int target, long long limit) {
   const long long t0 = clock64();
   while (tc::ld_acquire_smem(count) < target) {
     __nanosleep(64);  // leave the issue slots to the warps that are working
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
   return true;
 }
@@ -174,26 +223,28 @@ __device__ __forceinline__ bool count_wait_timeout(const int* count, int target)
 #define SLNR_TC_MBAR_SLEEP 256  // back-off (ns) between polls of an mbarrier by the MMA and epilogue warps
 #endif
 
-// Waits for the phase with the given parity to complete; false on timeout.
-// Sleeps between polls so that the waiting MMA and epilogue warps leave the
-// issue slots to the producers (their work has slack of a whole tile).
-__device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity) {
+// Waits for the phase with the given parity to complete; false after `limit`
+// clock cycles.  Sleeps between polls so that the waiting MMA and epilogue
+// warps leave the issue slots to the producers (their work has the slack of
+// a whole tile).
+__device__ __forceinline__ bool mbar_wait_timeout(uint64_t* bar, uint32_t parity, long long limit) {
   const long long t0 = clock64();
   while (!tc::mbar_try_wait(bar, parity)) {
     if (SLNR_TC_MBAR_SLEEP > 0) __nanosleep(SLNR_TC_MBAR_SLEEP);
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
   return true;
 }
 
 // Waits for the phase with the given parity to complete (1), or until
-// *end <= j, i.e. there is no tile j to wait for (0); -1 on timeout.
-__device__ __forceinline__ int mbar_wait_or_end(uint64_t* bar, uint32_t parity, const int* end, int j) {
+// *end <= j, i.e. there is no tile j to wait for (0); -1 after `limit` cycles.
+__device__ __forceinline__ int mbar_wait_or_end(uint64_t* bar, uint32_t parity, const int* end, int j,
+                                                long long limit) {
   const long long t0 = clock64();
   while (!tc::mbar_try_wait(bar, parity)) {
     if (*reinterpret_cast<const volatile int*>(end) <= j) return 0;
     if (SLNR_TC_MBAR_SLEEP > 0) __nanosleep(SLNR_TC_MBAR_SLEEP);
-    if (clock64() - t0 > kWaitCycles) return -1;
+    if (clock64() - t0 > limit) return -1;
   }
   return 1;
 }
@@ -217,146 +268,70 @@ __host__ __device__ constexpr int tc_nbuf(int K, int L) {
                    : 1;
 }
 
-// Shared memory: NBUF T tiles (kTcRows x KT) and D^T (L x KT), tf32 K-major
-// 128B-swizzled, plus 1 KB of alignment slack.
-__host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
-  return (size_t)tc_nbuf(K, L) * kTcRows * tc_kt(K) * 4 + (size_t)L * tc_kt(K) * 4 + 1024;
+// Epilogue staging: each of the four epilogue warps stages its 32 rows, one
+// column chunk of min(L, 32) values at a time, in shared memory with a row
+// pitch padded by 16 bytes (the warp's 16-byte stores of 32 different rows
+// then hit every bank evenly), and reads them back transposed so that each
+// global store instruction writes whole 128-byte row pieces: 4 rows of 32
+// values per instruction instead of 32 scattered 16-byte pieces (one lane
+// per row).  Two stages per warp where shared memory allows, else one.
+__host__ __device__ constexpr int tc_chunk(int L) { return L < 32 ? L : 32; }
+__host__ __device__ constexpr int tc_pitch(int L) { return tc_chunk(L) * 4 + 16; }
+__host__ __device__ constexpr size_t tc_stage_bytes(int L) { return (size_t)4 * 32 * tc_pitch(L); }
+__host__ __device__ constexpr size_t tc_td_bytes(int K, int L) {
+  return (size_t)tc_nbuf(K, L) * kTcRows * tc_kt(K) * 4 + (size_t)L * tc_kt(K) * 4;
+}
+__host__ __device__ constexpr int tc_nstage(int K, int L) {
+  return tc_td_bytes(K, L) + 2 * tc_stage_bytes(L) + 1024 <= (size_t)220 * 1024 ? 2 : 1;
 }
 
-#ifndef SLNR_TC_VPL
-#define SLNR_TC_VPL 4  // T-row columns per producer lane (4, 8 or 16)
-#endif
-#ifndef SLNR_TC_UNROLL
-#define SLNR_TC_UNROLL 8  // gathered rows in flight per lane group
-#endif
-#ifndef SLNR_TC_DENSE_ROWS
-#define SLNR_TC_DENSE_ROWS 4  // DENSE mode: rows of T loaded at once per lane group
-#endif
+// Shared memory: NBUF T tiles (kTcRows x KT) and D^T (L x KT), tf32 K-major
+// 128B-swizzled, then the epilogue stages, plus 1 KB of alignment slack.
+__host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
+  return tc_td_bytes(K, L) + tc_nstage(K, L) * tc_stage_bytes(L) + 1024;
+}
 
-// Producer layout: a T row is built by a group of GS = K / VPL lanes, lane gl
-// of the group holding the VPL columns [VPL*gl, VPL*gl + VPL), loaded as
-// float4s; a warp builds G = 32 / GS rows at once, one per group, with U row
-// gathers in flight per group.  A claim is the G consecutive items of one
-// warp pass.
-#ifndef SLNR_TC_TAIL_BATCH
-#define SLNR_TC_TAIL_BATCH 1  // segments without prefetch: the last batch loaded at once (0: row by row)
+#ifndef SLNR_TC_BATCH
+#define SLNR_TC_BATCH 4  // gathered rows a lane group keeps in flight (one batch; half with Hadamard rows)
 #endif
-#ifndef SLNR_TC_SEQ_SEGS
-#define SLNR_TC_SEQ_SEGS 2  // segments a lane group claims at once and gathers one after the other
-#endif
-#ifndef SLNR_TC_PF_AHEAD
-#define SLNR_TC_PF_AHEAD 8  // rows of a segment prefetched into L2 beyond the batch in flight
-#endif
+constexpr int kBatch = SLNR_TC_BATCH;
 
 // L2 prefetch of the 128-byte line holding p (no register, nothing to wait for).
 __device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 
-// acc += sum_{p in [p0,p1)} vals[p] * R(crd[p])[col .. col+VPL), sequential in p,
-// where R(k) = X[k,:] (or X[k,:] .* X2[k,:] with H).  U rows are loaded per
-// batch (the last batch predicated, so a short segment costs one round trip
-// per batch, not per row).  Rows further ahead are pulled into L2 by line
-// prefetches, which hold no register: each of the group's GS lanes prefetches
-// one 128-byte line, RPI = GS / LPR rows per step, and the front is kept AHEAD
-// rows beyond the batch in flight.
-template <int K, int VPL, int U, int AHEAD, bool H>
-__device__ __forceinline__ void gather_pf(float (&acc)[VPL], const int32_t* __restrict__ crd,
-                                          const float* __restrict__ vals, int p0, int p1,
-                                          const float* __restrict__ X, const float* __restrict__ X2, int col,
-                                          int gl) {
-  constexpr int GS = K / VPL, LPR = K >= 32 ? K / 32 : 1, RPI = GS / LPR;  // a row of 16 floats is half a line
-  static_assert(AHEAD % RPI == 0, "the prefetch window is whole steps");
-  constexpr int NPF = AHEAD / RPI;
-  const int prow = gl / LPR, poff = (gl % LPR) * 32;
-  auto pf_row = [&](int c) {
-    prefetch_line(X + (int64_t)c * K + poff);
-    if constexpr (H) prefetch_line(X2 + (int64_t)c * K + poff);
-  };
-  int pq = p0 + U;  // first row not covered by the first batch or the window
-  int pf = -1;      // coordinate of row pq + prow (the next prefetch step)
-  if constexpr (NPF > 0) {
-    int cs[NPF];
+// Producer lane layout: a T row is built by a group of GS = K / 4 lanes (at
+// most a warp), lane gl of the group holding the 4 columns [4 gl, 4 gl + 4)
+// as one float4; a warp holds G = 32 / GS groups.  A claim is IPC = G * R
+// consecutive items of an item tile, group g taking items g R .. g R + R - 1
+// (R more items per group where the rows are narrow, so a claim is at
+// least 8 items).
+template <int K>
+struct ProdLayout {
+  static constexpr int VPL = 4;
+  static constexpr int GS = K / VPL;
+  static constexpr int G = 32 / GS;
+  static constexpr int R = GS < kBatch ? GS : kBatch;
+  static constexpr int IPC = G * R;
+  static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
+  static_assert(kTcRows % IPC == 0, "claims tile the item tile");
+  static_assert(R <= GS, "each item record is held by one lane of its group");
+};
+
+// Row k of the gathered matrix, the VPL columns of this lane: X[k, col..] (or
+// X[k, col..] .* X2[k, col..] with H, the product formed in fp32).
+template <int K, int VPL, bool H>
+__device__ __forceinline__ void gathered_row(float (&x)[VPL], const float* __restrict__ X,
+                                             const float* __restrict__ X2, int c, int col) {
+  ldg_vec<VPL>(x, X + (int64_t)c * K + col);
+  if constexpr (H) {
+    float x2[VPL];
+    ldg_vec<VPL>(x2, X2 + (int64_t)c * K + col);
 #pragma unroll
-    for (int k = 0; k < NPF; ++k) {
-      const int q = pq + k * RPI + prow;
-      cs[k] = q < p1 ? __ldg(crd + q) : -1;
-    }
-    pq += AHEAD;
-    pf = pq + prow < p1 ? __ldg(crd + pq + prow) : -1;
-#pragma unroll
-    for (int k = 0; k < NPF; ++k)
-      if (cs[k] >= 0) pf_row(cs[k]);
-  }
-  // advances the prefetch front by one step when it is within AHEAD rows of p + U
-  auto advance = [&](int p) {
-    if constexpr (NPF > 0) {
-      if (pq < p + U + AHEAD && pq < p1) {
-        if (pf >= 0) pf_row(pf);
-        pq += RPI;
-        pf = pq + prow < p1 ? __ldg(crd + pq + prow) : -1;
-      }
-    }
-  };
-  auto row = [&](float (&x)[VPL], int c) {
-    ldg_vec<VPL>(x, X + (int64_t)c * K + col);
-    if constexpr (H) {
-      float x2[VPL];
-      ldg_vec<VPL>(x2, X2 + (int64_t)c * K + col);
-#pragma unroll
-      for (int e = 0; e < VPL; ++e) x[e] *= x2[e];
-    }
-  };
-  int p = p0;
-  for (; p + U <= p1; p += U) {  // full batches
-    advance(p);
-    int c[U];
-    float v[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      c[u] = __ldg(crd + p + u);
-      v[u] = __ldg(vals + p + u);
-    }
-    float x[U][VPL];
-#pragma unroll
-    for (int u = 0; u < U; ++u) row(x[u], c[u]);
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v[u], x[u][e], acc[e]);
-  }
-  if (p < p1) {  // the last, partial batch (all its loads still in flight together)
-    advance(p);
-    int c[U];
-    float v[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const bool ok = p + u < p1;
-      c[u] = ok ? __ldg(crd + p + u) : -1;
-      v[u] = ok ? __ldg(vals + p + u) : 0.f;
-    }
-    float x[U][VPL];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (c[u] >= 0) row(x[u], c[u]); else zero_vec(x[u]);
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (c[u] >= 0)
-#pragma unroll
-        for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v[u], x[u][e], acc[e]);
+    for (int e = 0; e < VPL; ++e) x[e] *= x2[e];
   }
 }
 
-template <int K>
-struct ProdLayout {
-  static constexpr int VPL = K / SLNR_TC_VPL >= 1 && K / SLNR_TC_VPL <= 32 ? SLNR_TC_VPL : 4;
-  static constexpr int GS = K / VPL;
-  static constexpr int G = 32 / GS;
-  static constexpr int U = SLNR_TC_UNROLL;
-  static_assert(VPL == 4 || VPL == 8 || VPL == 16, "VPL must be 4, 8 or 16");
-  static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
-};
-
-// Stores the VPL values of lane group column col of T row s (buffer sTb),
+// Stores the VPL values of this lane's columns of T row s (buffer sTb),
 // rounded to tf32, into the 128B-swizzled K-major tile.
 template <int VPL>
 __device__ __forceinline__ void store_t_part(uint8_t* sTb, int s, int col, const float (&acc)[VPL]) {
@@ -367,101 +342,342 @@ __device__ __forceinline__ void store_t_part(uint8_t* sTb, int s, int col, const
                    tc::to_tf32(acc[4 * h + 3]));
 }
 
-// Warp roles of the persistent tile kernel (32 warps):
-//   warps 0..26  producers: claim G consecutive items of this CTA's item
-//                tiles at a time (in order), build their T rows with one lane
-//                group per row, and store each row into its item's slot of
-//                the tile's T buffer with its destination; one mbarrier
-//                arrival per claim;
-//   warp 27      MMA issuer: waits full[b] (every claim of the tile placed)
-//                and free[b] (buffer's previous accumulator drained), issues
-//                the tile's K/8 tcgen05.mma into TMEM accumulator b, commits
-//                to mma[b];
-//   warps 28..31 epilogue: wait mma[b], read TMEM lane quadrant (warp % 4),
-//                write A rows or partial rows, arrive free[b].
-// Item tile n uses buffer n % NBUF; a producer stores into it only after the
-// MMAs of tile n - NBUF completed.  Claims are taken in order, so the claim a
-// producer waits on belongs to an earlier tile, which only needs earlier
-// claims (no cycle).  Producers wait on mma_tiles_done, a monotonic count of
-// completed tiles that the epilogue publishes (release) once all four
-// epilogue warps have read the tile's row destinations.  Every wait is
-// bounded; a timeout raises kErrTimeout and the CTA winds down.
-// Items per producer claim: SLNR_TC_SEQ_SEGS segments per lane group, or
-// SLNR_TC_DENSE_ROWS rows per lane group in DENSE mode.
-template <int K, int MODE>
-__host__ __device__ constexpr int claim_items() {
-  return ProdLayout<K>::G * (MODE == kDense ? SLNR_TC_DENSE_ROWS : SLNR_TC_SEQ_SEGS);
+// Segment record of item `item` ({row, p0, p1, partial slot}); items past the
+// list are {-1, 0, 0, -1}: no destination, no nonzeros.
+__device__ __forceinline__ int4 seg_rec(const int4* __restrict__ segs, int item, int nitems) {
+  return item < nitems ? __ldg(segs + item) : make_int4(-1, 0, 0, -1);
 }
 
-constexpr int kProducerWarps = 27;
+// The producer gathers below run in one lane group (GS lanes, mask gmask,
+// first lane gbase, this lane gl).  The group's R items are held one record
+// per lane: lane gl < R holds the p0 (rp0) and p1 (rp1) of item gl and its
+// destination (rdst: A row, partial slot).  Coordinates and values are loaded
+// cooperatively, one nonzero per lane, and handed to the gathering lanes with
+// shuffles inside the group.  Finished T rows are placed through `pl`
+// (completion-order slots, see the kernel): pl.take(n) returns the first of
+// n consecutive slots once their buffer is free (-1 after a timeout),
+// pl.put / pl.put_dest store a row and its destination, pl.publish(sl, n)
+// fences and arrives on the slot tiles' barriers.  Both return false after a
+// timeout.
+
+// A wave of W short items (items w0 .. w0 + W - 1, at most N nonzeros each,
+// W N <= kBatch): lane t loads the coordinate and value of slot t (nonzero
+// t % N of item t / N), all W N gathered rows are in flight at once, then
+// each item's T row is summed in nonzero order and placed.
+template <int K, int VPL, int GS, int W, int N, bool H, typename Place>
+__device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, int rp0, int rp1, int2 rdst, int w0,
+                                           const int32_t* __restrict__ crd, const float* __restrict__ vals,
+                                           const float* __restrict__ X, const float* __restrict__ X2, int col,
+                                           Place& pl) {
+  constexpr int S = W * N;                // row slots of the batch
+  constexpr int SPL = (S + GS - 1) / GS;  // slots loaded per lane
+  static_assert(S <= kBatch, "a wave is one batch");
+  int mc[SPL];
+  float mv[SPL];
+#pragma unroll
+  for (int h = 0; h < SPL; ++h) {
+    const int t = gl + h * GS, w = t / N < W ? t / N : W - 1, s = t % N;
+    const int p0 = __shfl_sync(gmask, rp0, gbase + w0 + w), p1 = __shfl_sync(gmask, rp1, gbase + w0 + w);
+    const bool ok = t < S && p0 + s < p1;
+    mc[h] = ok ? __ldg(crd + p0 + s) : -1;
+    mv[h] = ok ? __ldg(vals + p0 + s) : 0.f;
+  }
+  float x[S][VPL];
+#pragma unroll
+  for (int u = 0; u < S; ++u) {
+    const int c = __shfl_sync(gmask, mc[u / GS], gbase + u % GS);
+    if (c >= 0) gathered_row<K, VPL, H>(x[u], X, X2, c, col); else zero_vec(x[u]);
+  }
+  // each item's sum, in nonzero order, into the registers of its first row
+#pragma unroll
+  for (int w = 0; w < W; ++w)
+#pragma unroll
+    for (int s = 0; s < N; ++s) {
+      const int u = w * N + s;
+      const float v = __shfl_sync(gmask, mv[u / GS], gbase + u % GS);
+#pragma unroll
+      for (int e = 0; e < VPL; ++e) x[w * N][e] = s == 0 ? v * x[u][e] : fmaf(v, x[u][e], x[w * N][e]);
+    }
+  const int sl = pl.take(W);
+  if (sl < 0) return false;
+#pragma unroll
+  for (int w = 0; w < W; ++w) pl.put(sl + w, x[w * N]);
+  if (gl >= w0 && gl < w0 + W) pl.put_dest(sl + gl - w0, rdst);
+  pl.publish(sl, W);
+  return true;
+}
+
+// The group's R items one after the other, each T row summed in nonzero
+// order in batches of B gathered rows and placed when complete.  The items'
+// nonzeros are walked in chunks of GS (a chunk never spans two items): lane
+// t holds the coordinate and value of nonzero t of the current chunk, and the
+// next chunk's (which may be the next item's first) are loaded while this one
+// is gathered.  With PF the chunk after that is loaded too, and the rows of
+// the next chunk are prefetched into L2 (one lane per row,
+// prefetch.global.L2, no register held) while this chunk is gathered.
+template <int K, int VPL, int GS, int R, bool PF, bool H, typename Place>
+__device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, int rp0, int rp1, int2 rdst,
+                                           const int32_t* __restrict__ crd, const float* __restrict__ vals,
+                                           const float* __restrict__ X, const float* __restrict__ X2, int col,
+                                           Place& pl) {
+  constexpr int B0 = H ? kBatch / 2 : kBatch;  // two loads per nonzero with H
+  constexpr int B = B0 < GS ? B0 : GS;
+  static_assert(GS % B == 0, "batches tile a chunk");
+  constexpr int LPR = K * 4 / 128 > 0 ? K * 4 / 128 : 1;  // 128-byte lines per gathered row
+  auto p0_of = [&](int r) { return __shfl_sync(gmask, rp0, gbase + r); };
+  auto p1_of = [&](int r) { return __shfl_sync(gmask, rp1, gbase + r); };
+  // a chunk is item r's nonzeros [q, min(q + GS, p1(r))); r == R: none left
+  auto advance = [&](int& r, int& q) {
+    if (r < R && q + GS < p1_of(r)) {
+      q += GS;
+    } else {
+      ++r;
+      q = r < R ? p0_of(r) : 0;
+    }
+  };
+  auto load_idx = [&](int r, int q, int& ic, float& iv) {
+    const bool ok = r < R && q + gl < p1_of(r);
+    ic = ok ? __ldg(crd + q + gl) : -1;
+    iv = ok ? __ldg(vals + q + gl) : 0.f;
+  };
+  int r = 0, q = p0_of(0);  // current chunk
+  int rn = r, qn = q;       // next chunk
+  advance(rn, qn);
+  int r2 = rn, q2 = qn;     // the chunk after (PF)
+  if (PF) advance(r2, q2);
+  int ic, nc, n2c = -1;
+  float iv, nv, n2v = 0.f;
+  load_idx(r, q, ic, iv);
+  load_idx(rn, qn, nc, nv);
+  float acc[VPL];
+  zero_vec(acc);
+#pragma unroll 1
+  while (r < R) {
+    if constexpr (PF) {
+      if (nc >= 0)  // rows of the next chunk (coordinates loaded one chunk ago) into L2
+#pragma unroll
+        for (int l = 0; l < LPR; ++l) {
+          prefetch_line(X + (int64_t)nc * K + 32 * l);
+          if constexpr (H) prefetch_line(X2 + (int64_t)nc * K + 32 * l);
+        }
+      load_idx(r2, q2, n2c, n2v);  // two chunks ahead
+    }
+    const int m = min(GS, p1_of(r) - q);
+#pragma unroll 1
+    for (int u0 = 0; u0 < m; u0 += B) {
+      float x[B][VPL];
+#pragma unroll
+      for (int k = 0; k < B; ++k) {
+        const int c = __shfl_sync(gmask, ic, gbase + u0 + k);
+        if (c >= 0) gathered_row<K, VPL, H>(x[k], X, X2, c, col); else zero_vec(x[k]);
+      }
+#pragma unroll
+      for (int k = 0; k < B; ++k) {
+        const float v = __shfl_sync(gmask, iv, gbase + u0 + k);
+#pragma unroll
+        for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v, x[k][e], acc[e]);
+      }
+    }
+    if (rn != r) {  // the item's last chunk: its T row is complete
+      const int sl = pl.take(1);
+      if (sl < 0) return false;
+      pl.put(sl, acc);
+      if (gl == r) pl.put_dest(sl, rdst);
+      pl.publish(sl, 1);
+      zero_vec(acc);
+    }
+    r = rn;
+    q = qn;
+    ic = nc;
+    iv = nv;
+    if constexpr (PF) {
+      rn = r2;
+      qn = q2;
+      nc = n2c;
+      nv = n2v;
+      advance(r2, q2);
+    } else {
+      advance(rn, qn);
+      load_idx(rn, qn, nc, nv);
+    }
+  }
+  return true;
+}
+
 constexpr int kTileRing = 16;  // local tiles whose global index is kept in shared memory
-constexpr int kMmaWarp = 27;  // warps 28..31: epilogue
+constexpr int kMaxBuf = 4;     // T / accumulator buffers at most
+
+// Shared state of the tile kernel's pipeline (one per CTA; static shared
+// memory, named directly by the helpers below).
+struct TcShared {
+  uint64_t full_bar[kMaxBuf];  // slot tile b filled: one arrival per placed T row
+  uint64_t mma_bar[kMaxBuf];   // the tile's MMAs completed (tcgen05.commit)
+  uint64_t free_bar[kMaxBuf];  // the four epilogue warps have drained accumulator b
+  int2 dest[kMaxBuf][kTcRows]; // per slot: (A row, partial slot); x < 0 = no destination
+  uint32_t tmem_base;
+  int claim;                   // next producer claim of this CTA
+  int fill;                    // next T slot (completion order)
+  int fail_flag;               // a wait timed out: every role winds down
+  int epi_progress[4];         // per epilogue warp: tiles whose destinations it has read
+  int tile_gid[kTileRing];     // global item tile of local tile j (ring)
+  int tile_seq[kTileRing];     // j + 1 once tile_gid of local tile j is written
+  int end_tile;                // first local tile past the last item tile
+  int last_commit[kMaxBuf];    // last tile committed to each accumulator (-1: none)
+  float* epi_dst[4][32];       // per epilogue warp: destination of each of its 32 rows (nullptr: none)
+};
+__shared__ TcShared g_tc;
+extern __shared__ uint8_t smem_raw[];
+
+// Waits until every epilogue warp has read the destinations of `tiles` slot
+// tiles (each warp publishes its own count: a sum would let one warp that
+// runs ahead stand in for one that lags); false after `limit` clock cycles.
+__device__ __forceinline__ bool epi_wait_timeout(int tiles, long long limit) {
+  const long long t0 = clock64();
+  for (;;) {
+    int m = tc::ld_acquire_smem(&g_tc.epi_progress[0]);
+#pragma unroll
+    for (int q = 1; q < 4; ++q) m = min(m, tc::ld_acquire_smem(&g_tc.epi_progress[q]));
+    if (m >= tiles) return true;
+    __nanosleep(64);
+    if (clock64() - t0 > limit) return false;
+  }
+}
+
+// The T tiles: NBUF buffers at the first 1024-byte boundary of the dynamic
+// shared memory, then D^T.
+__device__ __forceinline__ uint8_t* tc_tiles() {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+}
+
+// Completion-order placement of one lane group's T rows: slots are taken
+// from the CTA's fill counter after the rows are built; slot s lives in slot
+// tile s / kTcRows, buffer (s / kTcRows) % NBUF.
+template <int VPL, int NBUF, int TBYTES>
+struct Placer {
+  unsigned gmask;
+  int gbase, gl, col;
+  long long wait_cycles;
+  // First of n consecutive slots, once the buffers of their slot tiles are
+  // free (all four epilogue warps have read the destinations of the tiles
+  // NBUF before, so those tiles' MMAs are done); -1 after a timeout.  A range
+  // may span two slot tiles.
+  __device__ __forceinline__ int take(int n) {
+    int sl = 0;
+    if (gl == 0) sl = atomicAdd(&g_tc.fill, n);
+    sl = __shfl_sync(gmask, sl, gbase);
+    const int tl = (sl + n - 1) / kTcRows;
+    if (tl >= NBUF) {
+      const bool ok = epi_wait_timeout(tl - NBUF + 1, wait_cycles);
+      if (__any_sync(gmask, !ok)) {
+        if (gl == 0) atomicOr(&g_tc.fail_flag, 1);
+        return -1;
+      }
+    }
+    return sl;
+  }
+  __device__ __forceinline__ void put(int slot, const float (&acc)[VPL]) {
+    store_t_part<VPL>(tc_tiles() + ((slot / kTcRows) % NBUF) * TBYTES, slot % kTcRows, col, acc);
+  }
+  __device__ __forceinline__ void put_dest(int slot, int2 d) { g_tc.dest[(slot / kTcRows) % NBUF][slot % kTcRows] = d; }
+  // The rows (and destinations) of slots [sl, sl + n) are stored: make them
+  // visible to the tensor cores and count them on their tiles' barriers.
+  __device__ __forceinline__ void publish(int sl, int n) {
+    tc::fence_proxy_async_smem();
+    __syncwarp(gmask);
+    if (gl == 0) {
+      const int n1 = min(n, kTcRows - sl % kTcRows);
+      tc::mbar_arrive_n(&g_tc.full_bar[(sl / kTcRows) % NBUF], (uint32_t)n1);
+      if (n > n1) tc::mbar_arrive_n(&g_tc.full_bar[(sl / kTcRows + 1) % NBUF], (uint32_t)(n - n1));
+    }
+  }
+};
+
+// Warp roles of the persistent tile kernel (kTcWarps warps):
+//   producers    (all but the last five warps): take claims of IPC
+//                consecutive items of this CTA's item tiles (in order) and
+//                build the items' T rows with one lane group per item; each
+//                finished row (or wave of short rows) takes the next T slots
+//                in completion order, waits until the slots' buffer is free,
+//                and is stored with its destination; one arrival per placed
+//                row on the slot tile's mbarrier (kTcRows per tile);
+//   MMA warp     waits full[b] (the slot tile is complete) and free[b] (the
+//                buffer's previous accumulator drained), issues the tile's
+//                K/8 tcgen05.mma into TMEM accumulator b, commits to mma[b];
+//   4 epilogue   wait mma[b], read their destinations and publish their own
+//   warps        progress (epi_progress), read their TMEM lane quadrant
+//                (warp % 4), stage the rows in shared memory and write them
+//                (A rows, or partial rows of heavy rows) with coalesced
+//                stores of whole row pieces, arrive free[b].
+// Slot tile j uses buffer j % NBUF; a row goes into it only after all four
+// epilogue warps have read the destinations of slot tile j - NBUF (so its
+// MMAs are done).  A CTA fills exactly as many slot tiles as it takes item
+// tiles (every item, padding included, takes one slot).  Slots are taken
+// after the rows are built, so a producer waits only for an earlier slot
+// tile, whose slots were all taken by warps that already hold their rows and
+// wait only for still earlier tiles: no cycle.  Every wait is bounded by
+// wait_cycles; a timeout raises kErrTimeout and the CTA winds down (MMAs
+// already issued are drained with the default limit before the tensor
+// memory is freed).
+constexpr int kProducerWarps = kTcWarps - 5;
+constexpr int kMmaWarp = kTcWarps - 5;  // then the four epilogue warps
 
 template <int K, int L, int MODE, bool PF>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_gemm(WsHeader* hdr, const int4* __restrict__ segs, int max_segs,
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
               const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ D,
-              float* __restrict__ A,
-              float* __restrict__ partial) {
+              float* __restrict__ A, float* __restrict__ partial, long long wait_cycles) {
   static_assert(K == 16 || K == 32 || K == 64 || K == 128, "K must be 16, 32, 64 or 128");
   static_assert(L % 16 == 0 && L >= 16 && L <= 256, "L must be a multiple of 16 in [16, 256]");
   constexpr int KT = tc_kt(K);  // tile columns (K, or 32 with zero padding)
-  static_assert(kTcThreads == 1024, "32 warps: 27 producers, 1 MMA, 4 epilogue");
   using PL = ProdLayout<K>;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
   constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
   constexpr int TBYTES = kTcRows * KT * 4;
-  extern __shared__ uint8_t smem_raw[];
-  __shared__ uint64_t full_bar[NBUF], mma_bar[NBUF], free_bar[NBUF];
-  __shared__ int2 dest[NBUF][kTcRows];  // per slot: (A row, partial slot); x < 0 = padding
-  __shared__ uint32_t tmem_base;
-  __shared__ int claim, fill, fail_flag, mma_tiles_done;
-  __shared__ int tile_gid[kTileRing], tile_seq[kTileRing], end_tile;
-  __shared__ int last_commit[NBUF];     // last tile committed to each accumulator (-1: none)
-  uint8_t* sT = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr int CPT = kTcRows / PL::IPC;  // claims per item tile
+  static_assert(NBUF <= kMaxBuf, "buffers");
+  uint8_t* sT = tc_tiles();
   uint8_t* sD = sT + NBUF * TBYTES;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (warp == kMmaWarp) {
-    tc::tmem_alloc(&tmem_base, NCOLS);
+    tc::tmem_alloc(&g_tc.tmem_base, NCOLS);
     tc::tmem_relinquish();
   }
   if (tid == 0) {
     for (int b = 0; b < NBUF; ++b) {
-      tc::mbar_init(&full_bar[b], kTcRows / claim_items<K, MODE>());  // one arrival per claim
-      tc::mbar_init(&mma_bar[b], 1);
-      tc::mbar_init(&free_bar[b], 4);
-      last_commit[b] = -1;
+      tc::mbar_init(&g_tc.full_bar[b], kTcRows);  // one arrival per placed T row
+      tc::mbar_init(&g_tc.mma_bar[b], 1);
+      tc::mbar_init(&g_tc.free_bar[b], 4);
+      g_tc.last_commit[b] = -1;
     }
     tc::fence_mbar_init();
-    claim = 0;
-    fill = 0;
-    fail_flag = 0;
-    mma_tiles_done = 0;
+    g_tc.claim = 0;
+    g_tc.fill = 0;
+    g_tc.fail_flag = 0;
+    for (int q = 0; q < 4; ++q) g_tc.epi_progress[q] = 0;
   }
   // Item tiles are handed out dynamically: CTAs take them from a global
   // counter in the workspace header (zeroed before the launch), one tile
-  // ahead of need, so the hub rows' costly tiles do not pile up on a few SMs.
-  // Local tile j's global index is published in a small shared ring
-  // (tile_gid, with tile_seq = j + 1 once written); the first local tile
-  // whose index lies past the last item tile is end_tile, and every role
-  // stops there.
-  int64_t nitems;
+  // ahead of need, so the costly tiles do not pile up on a few SMs.  Local
+  // tile j's global index is published in a small shared ring (g_tc.tile_gid,
+  // with g_tc.tile_seq = j + 1 once written); the first local tile whose index
+  // lies past the last item tile is g_tc.end_tile, and every role stops there.
+  int nitems;  // < 2^31: segments or rows
   if (MODE != kDense) {
     const int n = hdr->n_segs;
     nitems = n < max_segs ? n : max_segs;
   } else {
-    nitems = dense_rows;
+    nitems = (int)dense_rows;
   }
-  const int64_t ntiles = (nitems + kTcRows - 1) / kTcRows;
+  const int ntiles = (int)(((int64_t)nitems + kTcRows - 1) / kTcRows);
   if (tid == 0) {
-    for (int r = 0; r < kTileRing; ++r) tile_seq[r] = 0;
+    for (int r = 0; r < kTileRing; ++r) g_tc.tile_seq[r] = 0;
     const int g0 = atomicAdd(&hdr->next_tile, 1);
-    tile_gid[0] = g0;
-    tile_seq[0] = 1;
-    end_tile = g0 >= ntiles ? 0 : INT_MAX;
+    g_tc.tile_gid[0] = g0;
+    g_tc.tile_seq[0] = 1;
+    g_tc.end_tile = g0 >= ntiles ? 0 : INT_MAX;
   }
   // D (K x L, row-major) -> D^T as the B operand (L rows of KT), tf32; rows
   // k >= K of the padded tile are zero
@@ -484,159 +700,118 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   tc::tc_fence_before_sync();
   __syncthreads();
   tc::tc_fence_after_sync();
-  const uint32_t tmem = tmem_base;
+  const uint32_t tmem = g_tc.tmem_base;
 
   // global item tile of local tile t: >= 0 once known, -1 if t does not
-  // exist (t >= end_tile), -2 if the wait timed out
+  // exist (t >= g_tc.end_tile), -2 if the wait timed out
   auto tile_of = [&](int t) -> int {
     const long long t0 = clock64();
-    while (tc::ld_acquire_smem(&tile_seq[t % kTileRing]) != t + 1) {
-      if (*reinterpret_cast<volatile int*>(&end_tile) <= t) return -1;
+    while (tc::ld_acquire_smem(&g_tc.tile_seq[t % kTileRing]) != t + 1) {
+      if (*reinterpret_cast<volatile int*>(&g_tc.end_tile) <= t) return -1;
       __nanosleep(32);
-      if (clock64() - t0 > kWaitCycles) return -2;
+      if (clock64() - t0 > wait_cycles) return -2;
     }
-    const int gid = *reinterpret_cast<volatile int*>(&tile_gid[t % kTileRing]);
+    const int gid = *reinterpret_cast<volatile int*>(&g_tc.tile_gid[t % kTileRing]);
     return gid < ntiles ? gid : -1;
   };
-  // the first claim of local tile t fetches the global index of tile t + 1
+  // the first g_tc.claim of local tile t fetches the global index of tile t + 1
   auto fetch_next_tile = [&](int t) {
     const int gnext = atomicAdd(&hdr->next_tile, 1);
-    tile_gid[(t + 1) % kTileRing] = gnext;
-    if (gnext >= ntiles) atomicMin(&end_tile, t + 1);
-    tc::st_release_smem(&tile_seq[(t + 1) % kTileRing], t + 2);
+    g_tc.tile_gid[(t + 1) % kTileRing] = gnext;
+    if (gnext >= ntiles) atomicMin(&g_tc.end_tile, t + 1);
+    tc::st_release_smem(&g_tc.tile_seq[(t + 1) % kTileRing], t + 2);
   };
 
   if (warp < kProducerWarps) {
     // ---------------- producers ----------------
-    // A claim covers IPC = G * R consecutive items of local item tile c / CPT:
-    // lane group g builds the T rows of items g, g + G, ..., g + (R-1) G of
-    // the claim (R = 1 gathered segment, or R = U rows of a materialised T in
-    // DENSE mode, all loads in flight at once).  It builds the rows first,
-    // then waits for its buffer to be free (the MMAs of tile c / CPT - NBUF
-    // completed and their destinations read), stores the rows and their
-    // destinations, and lane 0 arrives once for the claim.
-    constexpr int VPL = PL::VPL, G = PL::G, R = MODE != kDense ? SLNR_TC_SEQ_SEGS : SLNR_TC_DENSE_ROWS;
-    constexpr int IPC = G * R, CPT = kTcRows / IPC;
-    static_assert(IPC == claim_items<K, MODE>(), "barrier count matches the claims");
-    static_assert(kTcRows % IPC == 0, "claims tile the item tile");
-    const int g = lane / PL::GS, col = (lane % PL::GS) * VPL;
-    // record of item g + r G of claim c, whose item tile has global index gid
-    auto load_rec = [&](int gid, int c, int r) -> int4 {
-      int4 rv = make_int4(-1, 0, 0, -1);
-      const int64_t item = (int64_t)gid * kTcRows + (c % CPT) * IPC + r * G + g;
-      if (item < nitems) rv = (MODE != kDense) ? __ldg(segs + item) : make_int4((int)item, 0, 0, -1);
-      return rv;
-    };
-    // takes the next claim of this CTA; returns its item tile's global index
-    // (< 0: no such tile / timeout).  The first claim of a local tile also
-    // fetches the next local tile's global index.
+    constexpr int VPL = PL::VPL, R = PL::R, GS = PL::GS;
+    const int g = lane / GS, gl = lane % GS, col = gl * VPL, gbase = g * GS;
+    const unsigned gmask = GS == 32 ? 0xffffffffu : (((1u << GS) - 1u) << gbase);
+    Placer<VPL, NBUF, TBYTES> pl{gmask, gbase, gl, col, wait_cycles};
     int known_tile = -1, known_gid = -1;  // the last local tile this warp resolved
-    auto take_claim = [&](int& c) -> int {
-      int v = 0;
-      if (lane == 0) v = atomicAdd(&claim, 1);
-      c = __shfl_sync(0xffffffffu, v, 0);
-      const int t = c / CPT;
-      if (t != known_tile) {
-        known_gid = __shfl_sync(0xffffffffu, tile_of(t), 0);
-        known_tile = known_gid >= 0 ? t : -1;
+    for (;;) {
+      int c = 0;
+      if (lane == 0) c = atomicAdd(&g_tc.claim, 1);
+      c = __shfl_sync(0xffffffffu, c, 0);
+      const int j = c / CPT;
+      if (j != known_tile) {
+        known_gid = __shfl_sync(0xffffffffu, tile_of(j), 0);
+        known_tile = known_gid >= 0 ? j : -1;
       }
       const int gid = known_gid;
-      if (gid >= 0 && c % CPT == 0) {
-        if (lane == 0) fetch_next_tile(t);
-        __syncwarp();
-      }
-      return gid;
-    };
-    int cl = 0;
-    int gid = take_claim(cl);
-    int4 rec = gid >= 0 ? load_rec(gid, cl, 0) : make_int4(-1, 0, 0, -1);  // segment record (R = 1)
-    while (gid >= 0) {
-      int cl_next = 0;
-      const int gid_next = take_claim(cl_next);
-      float acc[R][VPL];
-      int2 dst0 = make_int2(-1, -1);  // destination of the segment (R = 1)
-      if constexpr (MODE != kDense) {
-        // the group's R segments, one after the other (the first record was
-        // loaded with the previous claim; the others share its cache line)
-        int4 rr[R];
-        rr[0] = rec;
-#pragma unroll
-        for (int r = 1; r < R; ++r) rr[r] = load_rec(gid, cl, r);
-        const int4 rec_next = gid_next >= 0 ? load_rec(gid_next, cl_next, 0) : make_int4(-1, 0, 0, -1);
-        constexpr bool H = MODE == kSegmentsH;
-        constexpr int UG = H ? PL::U / 2 : PL::U;  // two loads per nonzero in Hadamard mode
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-          zero_vec(acc[r]);
-          if (rr[r].x >= 0) {
-            if constexpr (PF)
-              gather_pf<K, VPL, UG, SLNR_TC_PF_AHEAD, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, X2, col,
-                                                          lane % PL::GS);
-            else if constexpr (SLNR_TC_TAIL_BATCH)
-              gather_pf<K, VPL, UG, 0, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, X2, col, lane % PL::GS);
-            else
-              gather_acc<VPL, UG, H>(acc[r], crd, vals, rr[r].y, rr[r].z, X, K, col, X2);
-          }
-        }
-        dst0 = make_int2(rr[0].x, rr[0].w);
-        rec = rec_next;
-      } else {
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-          const int4 rr = load_rec(gid, cl, r);
-          if (rr.x >= 0) ldg_vec<VPL>(acc[r], X + (int64_t)rr.x * K + col); else zero_vec(acc[r]);
-        }
-      }
-      __syncwarp();
-      // the claim's IPC rows take the next IPC slots in completion order, so a
-      // long segment delays only its own rows, never a whole tile (the item
-      // tiles of this CTA, and the slot tiles the MMAs consume, are as many)
-      int sl = 0;
-      if (lane == 0) sl = atomicAdd(&fill, IPC);
-      sl = __shfl_sync(0xffffffffu, sl, 0);
-      const int j = sl / kTcRows, b = j % NBUF, s0 = sl % kTcRows + g;
-      if (j >= NBUF) {
-        const bool ok = count_wait_timeout(&mma_tiles_done, j - NBUF + 1);
-        if (!__all_sync(0xffffffffu, ok)) {
-          atomicOr(&fail_flag, 1);
-          break;
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < R; ++r) {
-        store_t_part<VPL>(sT + b * TBYTES, s0 + r * G, col, acc[r]);
-        if (lane % PL::GS == 0) {
-          if constexpr (MODE == kDense) {
-            dest[b][s0 + r * G] = make_int2(load_rec(gid, cl, r).x, -1);
-          } else if (r == 0) {
-            dest[b][s0] = dst0;
-          } else {
-            const int4 rq = load_rec(gid, cl, r);
-            dest[b][s0 + r * G] = make_int2(rq.x, rq.w);
-          }
-        }
-      }
-      tc::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&full_bar[b]);
-      if (gid_next == -2) {  // timed out waiting for a tile index
-        atomicOr(&fail_flag, 1);
+      if (gid < 0) {
+        if (gid == -2) atomicOr(&g_tc.fail_flag, 1);
         break;
       }
-      cl = cl_next;
-      gid = gid_next;
+      if (c % CPT == 0) {
+        if (lane == 0) fetch_next_tile(j);
+        __syncwarp();
+      }
+      if (*reinterpret_cast<volatile int*>(&g_tc.fail_flag) != 0) break;  // another role timed out
+      const int item0 = gid * kTcRows + (c % CPT) * PL::IPC + g * R;  // this group's first item
+      bool ok = true;
+      if constexpr (MODE == kDense) {
+        // R rows of the materialised T, all loads in flight at once
+        float x[R][VPL];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          if (item0 + r < nitems) ldg_vec<VPL>(x[r], X + (int64_t)(item0 + r) * K + col); else zero_vec(x[r]);
+        }
+        const int sl = pl.take(R);
+        ok = sl >= 0;
+        if (ok) {
+#pragma unroll
+          for (int r = 0; r < R; ++r) pl.put(sl + r, x[r]);
+          if (gl < R) pl.put_dest(sl + gl, make_int2(item0 + gl < nitems ? item0 + gl : -1, -1));
+          pl.publish(sl, R);
+        }
+      } else {
+        constexpr bool H = MODE == kSegmentsH;
+        // lane gl < R holds the record of the group's item gl
+        int rp0 = 0, rp1 = 0;
+        int2 rdst = make_int2(-1, -1);
+        if (gl < R) {
+          const int4 rec = seg_rec(segs, item0 + gl, nitems);
+          rp0 = rec.y;
+          rp1 = rec.z;
+          rdst = make_int2(rec.x, rec.w);
+        }
+        // The list is sorted by length class, longest first: no item after
+        // item0 has more nonzeros than item0's class bound, so item0 picks
+        // the wave shape for the group's R items.
+        constexpr int BW = H ? kBatch / 2 : kBatch;  // rows in flight per group (two loads each with H)
+        constexpr int W1 = R < BW ? R : BW;
+        constexpr int W2 = R < BW / 2 ? R : (BW / 2 > 1 ? BW / 2 : 1);
+        constexpr int W4 = R < BW / 4 ? R : (BW / 4 > 1 ? BW / 4 : 1);
+        const int n0 = __shfl_sync(gmask, rp1 - rp0, gbase);
+        if (n0 <= 1) {
+#pragma unroll 1
+          for (int w0 = 0; w0 < R && ok; w0 += W1)
+            ok = short_wave<K, VPL, GS, W1, 1, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
+        } else if (n0 <= 2) {
+#pragma unroll 1
+          for (int w0 = 0; w0 < R && ok; w0 += W2)
+            ok = short_wave<K, VPL, GS, W2, 2, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
+        } else if (n0 <= 4) {
+#pragma unroll 1
+          for (int w0 = 0; w0 < R && ok; w0 += W4)
+            ok = short_wave<K, VPL, GS, W4, 4, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
+        } else {
+          ok = long_items<K, VPL, GS, R, PF, H>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, col, pl);
+        }
+      }
+      if (!__all_sync(0xffffffffu, ok)) break;
     }
-    if (gid == -2) atomicOr(&fail_flag, 1);
   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t sT_addr = tc::smem_u32(sT), sD_addr = tc::smem_u32(sD);
       for (int j = 0;; ++j) {
         const int b = j % NBUF;
-        const int st = mbar_wait_or_end(&full_bar[b], (j / NBUF) & 1, &end_tile, j);
+        const int st = mbar_wait_or_end(&g_tc.full_bar[b], (j / NBUF) & 1, &g_tc.end_tile, j, wait_cycles);
         if (st == 0) break;  // this CTA has no tile j
-        if (st < 0 || (j >= NBUF && !mbar_wait_timeout(&free_bar[b], ((j / NBUF) - 1) & 1))) {
-          atomicOr(&fail_flag, 1);
+        if (st < 0 || (j >= NBUF && !mbar_wait_timeout(&g_tc.free_bar[b], ((j / NBUF) - 1) & 1, wait_cycles))) {
+          atomicOr(&g_tc.fail_flag, 1);
           break;
         }
         tc::tc_fence_after_sync();
@@ -649,65 +824,79 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const uint64_t bd = tc::desc_k_sw128(sD_addr + kb * L * 128 + ks * 32);
             tc::mma_tf32(tmem + (uint32_t)(b * L), ad, bd, IDESC, (kb | ks) != 0);
           }
-        tc::mma_commit(&mma_bar[b]);
-        last_commit[b] = j;
+        tc::mma_commit(&g_tc.mma_bar[b]);
+        g_tc.last_commit[b] = j;
       }
     }
     __syncwarp();
   } else {
     // ---------------- epilogue ----------------
     const int q = warp & 3;  // TMEM lane quadrant of this warp
+    constexpr int CW = tc_chunk(L), PITCH = tc_pitch(L), NSTAGE = tc_nstage(K, L);
+    uint8_t* stage = sT + tc_td_bytes(K, L) + (size_t)q * NSTAGE * 32 * PITCH;
+    int stage_i = 0;
     for (int j = 0;; ++j) {
       const int b = j % NBUF;
-      const int st = __shfl_sync(0xffffffffu, mbar_wait_or_end(&mma_bar[b], (j / NBUF) & 1, &end_tile, j), 0);
+      const int st =
+          __shfl_sync(0xffffffffu, mbar_wait_or_end(&g_tc.mma_bar[b], (j / NBUF) & 1, &g_tc.end_tile, j, wait_cycles), 0);
       if (st == 0) break;  // this CTA has no tile j
       if (st < 0) {
-        atomicOr(&fail_flag, 1);
+        atomicOr(&g_tc.fail_flag, 1);
         break;
       }
       tc::tc_fence_after_sync();
       const int rr = 32 * q + lane;
-      const int2 dd = dest[b][rr];
-      // all four epilogue warps have their destinations: the slot tile may be refilled
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (q == 0 && lane == 0) tc::st_release_smem(&mma_tiles_done, j + 1);
-      float* dst = nullptr;
-      if (dd.x >= 0) dst = dd.y < 0 ? A + (int64_t)dd.x * L : partial + (int64_t)dd.y * L;
-      if constexpr (L >= 32) {
+      const int2 dd = g_tc.dest[b][rr];
+      // this warp has its destinations: once all four have, the slot tile may be refilled
+      __syncwarp();
+      if (lane == 0) tc::st_release_smem(&g_tc.epi_progress[q], j + 1);
+      // the destinations of the warp's 32 rows, read back by the lanes that
+      // store each row piece
+      constexpr int LPRW = CW / 4, RPI = 32 / LPRW, NIT = 32 / RPI;
+      g_tc.epi_dst[q][lane] =
+          dd.x < 0 ? nullptr : (dd.y < 0 ? A + (int64_t)dd.x * L : partial + (int64_t)dd.y * L);
+      __syncwarp();
+      // each chunk of CW columns: TMEM -> registers (row `lane`) -> this
+      // warp's stage -> 16-byte pieces of whole row pieces -> global
 #pragma unroll 1
-        for (int c = 0; c < L; c += 32) {
-          float v[32];
+      for (int c = 0; c < L; c += CW) {
+        float v[CW];
+        if constexpr (CW == 32)
           tc::tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
-          if (dst != nullptr) {
-            float4* o = reinterpret_cast<float4*>(dst + c);
+        else
+          tc::tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L + c), v);
+        uint8_t* st = stage + (size_t)stage_i * 32 * PITCH;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          }
-        }
-      } else {
-        float v[16];
-        tc::tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * L), v);
-        if (dst != nullptr) {
-          float4* o = reinterpret_cast<float4*>(dst);
+        for (int i = 0; i < CW / 4; ++i)
+          *reinterpret_cast<float4*>(st + (size_t)lane * PITCH + 16 * i) =
+              make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        __syncwarp();
 #pragma unroll
-          for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        for (int i = 0; i < NIT; ++i) {
+          const int r = RPI * i + lane / LPRW, part = lane % LPRW;
+          const float4 x = *reinterpret_cast<const float4*>(st + (size_t)r * PITCH + 16 * part);
+          float* d = g_tc.epi_dst[q][r];
+          if (d != nullptr) *reinterpret_cast<float4*>(d + c + 4 * part) = x;
         }
+        stage_i = (stage_i + 1) % NSTAGE;  // with one stage, the next chunk's
+        if (NSTAGE == 1) __syncwarp();     // stores wait for these reads
       }
       tc::tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&free_bar[b]);
+      if (lane == 0) tc::mbar_arrive(&g_tc.free_bar[b]);
     }
   }
 
   // ---- teardown: every role has finished its loop
   tc::tc_fence_before_sync();
   __syncthreads();
-  if (fail_flag) {
-    // MMAs of abandoned tiles may still be running: wait (bounded) for each
-    // accumulator's last commit before the tensor memory is released
+  if (g_tc.fail_flag) {
+    // MMAs of abandoned tiles may still be running: wait (bounded, with the
+    // default limit whatever wait_cycles was) for each accumulator's last
+    // commit before the tensor memory is released
     if (warp == kMmaWarp && lane == 0)
       for (int b = 0; b < NBUF; ++b)
-        if (last_commit[b] >= 0) mbar_wait_timeout(&mma_bar[b], (last_commit[b] / NBUF) & 1);
+        if (g_tc.last_commit[b] >= 0) mbar_wait_timeout(&g_tc.mma_bar[b], (g_tc.last_commit[b] / NBUF) & 1, kWaitCycles);
     if (tid == 0) atomicOr(&hdr->error, kErrTimeout);
   }
   __syncthreads();
@@ -761,6 +950,7 @@ template <int MODE, bool PF>
 cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const int4* segs,
                         int max_segs, int64_t dense_rows, const int32_t* crd, const float* vals, const float* X,
                         const float* X2, const float* D, float* A, float* partial, cudaStream_t s) {
+  const long long wait = wait_limit_cycles();
 #define SLNR_TC_CASE(KK, LL)                                                                              \
   if (K == KK && L == LL) {                                                                               \
     TcLaunch tl;                                                                                          \
@@ -772,7 +962,7 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
     if ((e = cudaMemsetAsync(&hdr->next_tile, 0, sizeof(int), s)) != cudaSuccess) return e;               \
     k_tc_gemm<KK, LL, MODE, PF><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,          \
                                                                              dense_rows, crd, vals, X,    \
-                                                                             X2, D, A, partial);          \
+                                                                             X2, D, A, partial, wait);    \
     return cudaGetLastError();                                                                            \
   }
   SLNR_TC_CASE(16, 16) SLNR_TC_CASE(16, 32) SLNR_TC_CASE(16, 64) SLNR_TC_CASE(16, 128) SLNR_TC_CASE(16, 256)
@@ -800,7 +990,7 @@ size_t l2_bytes() {
 
 bool tc_supported(int K, int L) {
   return (K == 16 || K == 32 || K == 64 || K == 128) && (L == 16 || L == 32 || L == 64 || L == 128 || L == 256) &&
-         tc_smem_bytes(K, L) <= (size_t)200 * 1024;
+         tc_smem_bytes(K, L) <= (size_t)220 * 1024;
 }
 
 int seg_scan_blocks(int64_t nrows) { return (int)((nrows + kScanRows - 1) / kScanRows); }
@@ -823,7 +1013,7 @@ cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, 
                                 const SegPlan& plan, cudaStream_t s, const float* C2) {
   if (B.nrows <= 0) return cudaSuccess;
   // Gathered rows that do not fit in half of L2 miss often: the producers
-  // then prefetch the rows ahead of their gathers into L2 (gather_pf).
+  // then prefetch the rows of the next chunk of nonzeros into L2 (long_items).
   const bool pf = (size_t)B.ncols * (size_t)K * sizeof(float) * (C2 != nullptr ? 2 : 1) > l2_bytes() / 2;
   if (C2 != nullptr)
     return pf ? tc_dispatch<kSegmentsH, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
