@@ -515,8 +515,7 @@ slnr_status slnr_sddmm_spmm(const slnr_csr* B, const float* C, const float* D, i
   const SplitPlan sp = split_plan(ws, l);
   SLNR_LAUNCH("classify", launch_classify(v, sp, s));
   if (opts->variant == SLNR_FUSED) {
-    SLNR_LAUNCH("sddmm_spmm_chunks", launch_sddmm_spmm_chunks(v, C, D, L, E, K, sp, s));
-    SLNR_LAUNCH("sddmm_spmm_rows", launch_sddmm_spmm_rows(v, C, D, L, E, K, A, sp.hdr, s));
+    SLNR_LAUNCH("sddmm_spmm_rows", launch_sddmm_spmm_rows(v, C, D, L, E, K, A, sp, s));
     SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, A, s));
   } else {
     float* Y = reinterpret_cast<float*>(ws + l.o_inter);

@@ -62,11 +62,15 @@ struct SliceUnits {      // MTTKRP: units of one slice
   int count;
 };
 
-struct Unit {            // MTTKRP: window `u` of slice `slice`, fibers [flo, fhi)
+struct Unit {            // MTTKRP: window `u` of slice `slice`
   int slice;
   int u;
-  int flo;
+  int flo;               // fibers starting in the window: [flo, fhi)
   int fhi;
+  int p0;                // the window's nonzeros: [p0, p1)
+  int p1;
+  int ffirst;            // the fiber holding nonzero p0 (the last whose first nonzero is <= p0)
+  int pad;
 };
 
 // Validation flag bits

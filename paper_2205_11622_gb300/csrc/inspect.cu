@@ -80,12 +80,13 @@ __global__ void k_csf_units(int nslices, const int32_t* __restrict__ pos2,
       continue;
     }
     if (lane == 0) su[s] = SliceUnits{base, nu};
-    for (int u = lane; u < nu; u += 32) units[base + u] = Unit{s, u, 0, 0};
+    for (int u = lane; u < nu; u += 32) units[base + u] = Unit{s, u, 0, 0, 0, 0, 0, 0};
   }
 }
 
-// One thread per unit: its fiber range [flo, fhi), the fibers of its slice
-// whose first nonzero lies in the unit's window (binary searches over pos3).
+// One thread per unit: its nonzero window [p0, p1), the fiber holding p0,
+// and the fibers of its slice whose first nonzero lies in the window
+// [flo, fhi) (binary searches over pos3).
 __global__ void k_unit_ranges(const WsHeader* __restrict__ hdr, int max_units, const int32_t* __restrict__ pos2,
                               const int32_t* __restrict__ pos3, const SliceUnits* __restrict__ su,
                               Unit* __restrict__ units) {
@@ -97,6 +98,11 @@ __global__ void k_unit_ranges(const WsHeader* __restrict__ hdr, int max_units, c
     const int lo_key = start + un.u * kUnitNnz;
     un.flo = un.u == 0 ? f0 : lower_bound_pos(pos3, f0, f1, lo_key);
     un.fhi = un.u == count - 1 ? f1 : lower_bound_pos(pos3, f0, f1, lo_key + kUnitNnz);
+    const int end = pos3[f1];
+    un.p0 = min(lo_key, end);
+    un.p1 = un.u == count - 1 ? end : min(lo_key + kUnitNnz, end);
+    // the fiber holding p0: flo if it starts exactly there, else the one before
+    un.ffirst = (un.flo < f1 && pos3[un.flo] == un.p0) || un.flo == f0 ? un.flo : un.flo - 1;
     units[w] = un;
   }
 }

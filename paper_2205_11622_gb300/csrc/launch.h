@@ -102,9 +102,10 @@ cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const 
                                  WsHeader* hdr, cudaStream_t s);
 
 // sddmm.cu
-// (hdr->next_row must be 0: warps take rows from it)
+// fused <SDDMM,SpMM>: the heavy rows' chunks (partials) and the light rows in
+// one launch (plan.hdr->next_row must be 0: warps take work from it)
 cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float* D, int L,
-                                   const float* E, int K, float* A, WsHeader* hdr, cudaStream_t s);
+                                   const float* E, int K, float* A, const SplitPlan& plan, cudaStream_t s);
 cudaError_t launch_sddmm_spmm_chunks(const CsrView& B, const float* C, const float* D, int L,
                                      const float* E, int K, const SplitPlan& plan, cudaStream_t s);
 // fused <SDDMM,SpMM,GEMM> over light rows: C nrows x K, D ncols x K, F ncols x L, W L x M

@@ -15,15 +15,41 @@
 #include "launch.h"
 
 #ifndef SLNR_MTTKRP_MIN_CTAS
-#define SLNR_MTTKRP_MIN_CTAS 5  // resident 256-thread CTAs per SM the unit kernel is compiled for (48 registers)
+#define SLNR_MTTKRP_MIN_CTAS 4  // resident 256-thread CTAs per SM the unit kernel is compiled for (64 registers)
 #endif
 #ifndef SLNR_MTTKRP_U
-#define SLNR_MTTKRP_U 4  // nonzeros of a fiber in flight per lane group
+#define SLNR_MTTKRP_U 4  // nonzeros a lane group gathers at once (each a D row and, at a fiber's end, a C row)
 #endif
 
 namespace slnr {
 namespace {
 
+// Lane layout of the fused unit kernel: a gathered row of L values is read by
+// a group of GS lanes (VPL columns each), a warp holds G groups.
+template <int L>
+struct FlatLanes {
+  static constexpr int VPL = L >= 256 ? 8 : 4;
+  static constexpr int GS = L / VPL;
+  static constexpr int G = 32 / GS;
+  static constexpr int B = 32 / G;                       // nonzeros per group per warp step
+  static constexpr int UB0 = VPL == 8 ? SLNR_MTTKRP_U / 2 : SLNR_MTTKRP_U;  // same registers for wide rows
+  static constexpr int UB = B < UB0 ? B : UB0;           // of those, gathered at once
+  static_assert(GS >= 1 && GS <= 32 && B % UB == 0, "lane layout");
+};
+
+// Fused MTTKRP over units (windows of at most kUnitNnz consecutive nonzeros
+// of one slice), nonzero-parallel: a warp takes a unit and walks its
+// nonzeros in steps of 32, lane l holding nonzero q + l (coordinate and
+// value loaded coalesced).  The fibers those nonzeros belong to come from a
+// coalesced window of the next 32 fiber starts: each lane counts the starts
+// at or before its nonzero (a binary search over the window by shuffles), so
+// no load waits for another load of the same step.  Lane group g then
+// gathers the D rows of nonzeros g B .. g B + B - 1, sums each fiber's run in
+// nonzero order (the producer, T(l) = sum_k B(i,j,k) D(k,l)) and, where the
+// run ends, multiplies it by C(j,:) and adds it to the unit's partial row
+// (the consumer).  A fiber that spans groups or steps contributes one run
+// per piece, which by linearity adds up to its T times C(j,:).  The order is
+// fixed by the data, so results are the same on every run.
 template <int L>
 __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(WsHeader* __restrict__ hdr,
                                                       const Unit* __restrict__ units,
@@ -36,65 +62,74 @@ __global__ void __launch_bounds__(256, SLNR_MTTKRP_MIN_CTAS) k_mttkrp_units(WsHe
                                                       const float* __restrict__ C,
                                                       const float* __restrict__ D,
                                                       float* __restrict__ partial) {
-  using RL = RowLanes<L>;
+  using FL = FlatLanes<L>;
+  constexpr int VPL = FL::VPL, GS = FL::GS, B = FL::B, UB = FL::UB;
+  constexpr unsigned FULL = 0xffffffffu;
   const int n = min(hdr->n_units, max_units);
-  const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
-  // warps take units one at a time from the header's counter (units of hub
-  // slices hold far more work than those of small slices)
+  const int lane = threadIdx.x & 31, g = lane / GS, col = (lane % GS) * VPL;
   for (;;) {
     int w = 0;
     if (lane == 0) w = atomicAdd(&hdr->next_unit, 1);
-    w = __shfl_sync(0xffffffffu, w, 0);
+    w = __shfl_sync(FULL, w, 0);
     if (w >= n) break;
     const Unit un = units[w];
-    const int flo = un.flo, fhi = un.fhi;  // fibers starting in the unit's window (inspector)
-    float acc[RL::VPL];
+    const int hi = un.p1, f1 = __ldg(pos2 + un.slice + 1);
+    int q = un.p0, fcur = un.ffirst;  // pos3[fcur] <= q
+    float acc[VPL];
     zero_vec(acc);
-    // The group's fibers f = flo + grp + n GPW, software-pipelined in three
-    // stages so that one round trip serves three fibers: with fiber f's rows
-    // in flight, the first nonzero (k, value) of fiber f + GPW and the record
-    // (pos3 range, j) of fiber f + 2 GPW are loaded.  Most fibers have one
-    // nonzero, whose D row then needs no further dependent load.
-    constexpr int GPW = RL::GPW;
-    auto load_rec = [&](int f, int& p0, int& p1, int& j) {
-      if (f < fhi) { p0 = __ldg(pos3 + f); p1 = __ldg(pos3 + f + 1); j = __ldg(crd2 + f); }
-      else { p0 = 0; p1 = 0; j = 0; }
-    };
-    auto load_first = [&](int p0, int p1, int& k, float& v) {
-      if (p0 < p1) { k = __ldg(crd3 + p0); v = __ldg(vals + p0); }
-      else { k = -1; v = 0.f; }
-    };
-    int f = flo + grp;
-    int p0a, p1a, ja, p0b, p1b, jb, ka;
-    float va;
-    load_rec(f, p0a, p1a, ja);
-    load_rec(f + GPW, p0b, p1b, jb);
-    load_first(p0a, p1a, ka, va);
-    for (; f < fhi; f += GPW) {
-      int kb, p0c, p1c, jc;
-      float vb;
-      load_first(p0b, p1b, kb, vb);
-      load_rec(f + 2 * GPW, p0c, p1c, jc);
-      float c[RL::VPL];
-      ldg_vec<RL::VPL>(c, C + (int64_t)ja * L + col);
-      // producer: T(l) = sum_k B(i,j,k) D(k,l), in registers, in nonzero order
-      float t[RL::VPL];
+    while (q < hi) {  // warp-uniform
+      // the window: starts of fibers fcur + 1 .. fcur + 32 (past the slice: never)
+      const int fm = fcur + 1 + lane;
+      const int s = fm < f1 ? __ldg(pos3 + fm) : INT_MAX;
+      const int jn = fm < f1 ? __ldg(crd2 + fm) : 0;
+      const int j0 = __ldg(crd2 + fcur);
+      const int qe = min(min(q + 32, hi), __shfl_sync(FULL, s, 31));  // labels stay inside the window
+      const int p = q + lane;
+      const bool live = p < qe;
+      const int kk = live ? __ldg(crd3 + p) : 0;
+      const float vv = live ? __ldg(vals + p) : 0.f;
+      // cnt = starts at or before p (s is sorted): p is in fiber fcur + cnt
+      int cnt = 0;
+#pragma unroll
+      for (int step = 16; step > 0; step >>= 1)
+        if (__shfl_sync(FULL, s, cnt + step - 1) <= p) cnt += step;
+      const int jx = __shfl_sync(FULL, jn, cnt > 0 ? cnt - 1 : 0);
+      const int jj = cnt > 0 ? jx : j0;
+      const int cprev = __shfl_up_sync(FULL, cnt, 1), cnext = __shfl_down_sync(FULL, cnt, 1);
+      const bool start = lane % B == 0 || cprev != cnt;
+      const bool end = live && (lane % B == B - 1 || p + 1 >= qe || cnext != cnt);
+      const int flags = (start ? 1 : 0) | (end ? 2 : 0) | (live ? 4 : 0);
+      // group g: its B nonzeros in order, UB at a time
+      float t[VPL];
       zero_vec(t);
-      if (ka >= 0) {
-        float x[RL::VPL];
-        ldg_vec<RL::VPL>(x, D + (int64_t)ka * L + col);
 #pragma unroll
-        for (int e = 0; e < RL::VPL; ++e) t[e] = fmaf(va, x[e], t[e]);
-        gather_acc<RL::VPL, SLNR_MTTKRP_U>(t, crd3, vals, p0a + 1, p1a, D, L, col);
+      for (int u0 = 0; u0 < B; u0 += UB) {
+        float x[UB][VPL], cr[UB][VPL], v[UB];
+        int fl[UB];
+#pragma unroll
+        for (int k = 0; k < UB; ++k) {
+          const int l = g * B + u0 + k;
+          const int ck = __shfl_sync(FULL, kk, l), jk = __shfl_sync(FULL, jj, l);
+          v[k] = __shfl_sync(FULL, vv, l);
+          fl[k] = __shfl_sync(FULL, flags, l);
+          if (fl[k] & 4) ldg_vec<VPL>(x[k], D + (int64_t)ck * L + col); else zero_vec(x[k]);
+          if (fl[k] & 2) ldg_vec<VPL>(cr[k], C + (int64_t)jk * L + col); else zero_vec(cr[k]);
+        }
+#pragma unroll
+        for (int k = 0; k < UB; ++k) {
+#pragma unroll
+          for (int e = 0; e < VPL; ++e) t[e] = fmaf(v[k], x[k][e], (fl[k] & 1) ? 0.f : t[e]);
+          if (fl[k] & 2)
+#pragma unroll
+            for (int e = 0; e < VPL; ++e) acc[e] = fmaf(t[e], cr[k][e], acc[e]);
+        }
       }
-      // consumer: A(i,l) += T(l) C(j,l)
-#pragma unroll
-      for (int x = 0; x < RL::VPL; ++x) acc[x] = fmaf(t[x], c[x], acc[x]);
-      p0a = p0b; p1a = p1b; ja = jb; ka = kb; va = vb;
-      p0b = p0c; p1b = p1c; jb = jc;
+      // the next step starts in the fiber holding qe
+      fcur += __popc(__ballot_sync(FULL, s <= qe));
+      q = qe;
     }
-    cross_group_sum<RL::GS>(acc);
-    if (grp == 0) st_vec(partial + w * L + col, acc);
+    cross_group_sum<GS>(acc);
+    if (g == 0) st_vec(partial + (int64_t)w * L + col, acc);
   }
 }
 

@@ -18,6 +18,7 @@
 #define SLNR_SDDMM_MIN_CTAS 4  // resident 256-thread CTAs per SM the fused kernels are compiled for (64 registers)
 #endif
 constexpr int kRowsPerClaim = 4;  // rows a warp of the fused row kernel takes at a time
+constexpr int kShortRow = 8;      // a claim whose rows all have at most this many nonzeros: a lane group per row
 
 #ifndef SLNR_SDDMM_U
 #define SLNR_SDDMM_U 2  // nonzeros in flight per lane group
@@ -71,6 +72,55 @@ __device__ __forceinline__ void sddmm_spmm_range(float (&acc)[RowLanes<WM>::VPL]
   }
 }
 
+// One launch for all of a call's work: warps take items from the header's
+// counter, first the chunks of heavy rows (partial A rows into the
+// workspace, summed later by k_combine), then blocks of kRowsPerClaim light
+// rows (A rows written once).  Row lengths follow a power law, so the
+// costly hub chunks start first and every warp stays busy until the counter
+// runs out.
+// A row of at most kShortRow nonzeros owned by one lane group: for each
+// nonzero in order, acc += vals[p] <c, D(crd[p], :)> E(crd[p], :), U nonzeros
+// in flight.  The trip count is the warp's longest row (maxlen, the same in
+// every lane: the dot products' shuffles need the whole warp); shorter rows'
+// slots are predicated off.
+template <int WM, int U = SLNR_SDDMM_U>
+__device__ __forceinline__ void short_row_range(float (&acc)[RowLanes<WM>::VPL],
+                                                const float (&c)[RowLanes<WM>::VPL], int p0, int p1, int maxlen,
+                                                const int32_t* __restrict__ crd, const float* __restrict__ vals,
+                                                const float* __restrict__ D, int L, const float* __restrict__ E,
+                                                int K, int col) {
+  using RL = RowLanes<WM>;
+  constexpr int VPL = RL::VPL;
+  for (int it = 0; it < maxlen; it += U) {
+    const int base = p0 + it;
+    int cc[U];
+    float vv[U];
+    bool ok[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      ok[u] = base + u < p1;
+      cc[u] = ok[u] ? __ldg(crd + base + u) : 0;
+      vv[u] = ok[u] ? __ldg(vals + base + u) : 0.f;
+    }
+    float d[U][VPL], e[U][VPL];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (ok[u] && col < L) ldg_vec_upto<VPL>(d[u], D + (int64_t)cc[u] * L + col, L - col); else zero_vec(d[u]);
+      if (ok[u] && col < K) ldg_vec_upto<VPL>(e[u], E + (int64_t)cc[u] * K + col, K - col); else zero_vec(e[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      float dot = 0.f;
+#pragma unroll
+      for (int x = 0; x < VPL; ++x) dot = fmaf(c[x], d[u][x], dot);
+      dot = group_sum<RL::GS>(dot);
+      const float y = vv[u] * dot;
+#pragma unroll
+      for (int x = 0; x < VPL; ++x) acc[x] = fmaf(y, e[u][x], acc[x]);
+    }
+  }
+}
+
 template <int WM>
 __global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_rows(WsHeader* hdr, int nrows,
                                                                               const int32_t* __restrict__ pos,
@@ -79,21 +129,51 @@ __global__ void __launch_bounds__(256, SLNR_SDDMM_MIN_CTAS) k_sddmm_spmm_rows(Ws
                                                                               const float* __restrict__ C,
                                                                               const float* __restrict__ D, int L,
                                                                               const float* __restrict__ E, int K,
-                                                                              float* __restrict__ A) {
+                                                                              float* __restrict__ A,
+                                                                              const Chunk* __restrict__ chunks,
+                                                                              int max_chunks,
+                                                                              float* __restrict__ partial) {
   using RL = RowLanes<WM>;
   const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
-  // warps take blocks of kRowsPerClaim rows from the header's counter until
-  // the rows run out (row lengths follow a power law: static assignment
-  // leaves warps, and the CTAs holding them, idle)
+  const int nch = min(hdr->n_chunks, max_chunks);
   for (;;) {
-    int r0 = 0;
-    if (lane == 0) r0 = atomicAdd(&hdr->next_row, kRowsPerClaim);
-    r0 = __shfl_sync(0xffffffffu, r0, 0);
+    int w = 0;
+    if (lane == 0) w = atomicAdd(&hdr->next_row, 1);
+    w = __shfl_sync(0xffffffffu, w, 0);
+    if (w < nch) {  // a chunk of a heavy row
+      const Chunk ch = chunks[w];
+      float c[RL::VPL], acc[RL::VPL];
+      if (col < L) ldg_vec_upto<RL::VPL>(c, C + (int64_t)ch.row * L + col, L - col); else zero_vec(c);
+      zero_vec(acc);
+      sddmm_spmm_range<WM>(acc, c, ch.p0, ch.p1, crd, vals, D, L, E, K, grp, col);
+      cross_group_sum<RL::GS>(acc);
+      if (grp == 0 && col < K) st_vec_upto(partial + (int64_t)ch.slot * K + col, acc, K - col);
+      continue;
+    }
+    const int64_t r0 = (int64_t)(w - nch) * kRowsPerClaim;
     if (r0 >= nrows) break;
-    const int r1 = r0 + kRowsPerClaim < nrows ? r0 + kRowsPerClaim : nrows;
+    const int64_t r1 = r0 + kRowsPerClaim < nrows ? r0 + kRowsPerClaim : nrows;
+    // short rows: one row per lane group (no cross-group sum), nonzeros in order
+    if constexpr (RL::GPW >= kRowsPerClaim) {
+      const int64_t rg = r0 + grp;
+      int gp0 = 0, gp1 = 0;
+      if (grp < kRowsPerClaim && rg < r1) {
+        gp0 = pos[rg];
+        gp1 = pos[rg + 1];
+      }
+      const int maxlen = __reduce_max_sync(0xffffffffu, gp1 - gp0);
+      if (maxlen <= kShortRow) {  // warp-uniform
+        float c[RL::VPL], acc[RL::VPL];
+        zero_vec(acc);
+        if (gp1 > gp0 && col < L) ldg_vec_upto<RL::VPL>(c, C + rg * L + col, L - col); else zero_vec(c);
+        short_row_range<WM>(acc, c, gp0, gp1, maxlen, crd, vals, D, L, E, K, col);
+        if (grp < kRowsPerClaim && rg < r1 && col < K) st_vec_upto(A + rg * K + col, acc, K - col);
+        continue;
+      }
+    }
     for (int64_t r = r0; r < r1; ++r) {
       const int p0 = pos[r], p1 = pos[r + 1];
-      if (p1 - p0 > kLightMax) continue;  // warp-uniform
+      if (p1 - p0 > kLightMax) continue;  // warp-uniform: its chunks above
       float c[RL::VPL], acc[RL::VPL];
       if (col < L) ldg_vec_upto<RL::VPL>(c, C + r * L + col, L - col); else zero_vec(c);
       zero_vec(acc);
@@ -247,15 +327,16 @@ inline int grid_rows(int64_t nwarps_needed) {
 }  // namespace
 
 cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float* D, int L,
-                                   const float* E, int K, float* A, WsHeader* hdr, cudaStream_t s) {
+                                   const float* E, int K, float* A, const SplitPlan& plan, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
   const int WM = L > K ? L : K;
   // as many CTAs as stay resident; hdr->next_row starts at 0 (header zeroed by the call)
-  int64_t ctas = ceil_div(ceil_div(B.nrows, kRowsPerClaim), 8);
+  int64_t ctas = ceil_div(ceil_div(B.nrows, kRowsPerClaim) + plan.max_chunks, 8);
   const int64_t cap = (int64_t)device_sm_count() * SLNR_SDDMM_MIN_CTAS;
   if (ctas > cap) ctas = cap;
   SLNR_WIDTH_SWITCH(WM, W, {
-    k_sddmm_spmm_rows<W><<<(unsigned)ctas, 256, 0, s>>>(hdr, B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A);
+    k_sddmm_spmm_rows<W><<<(unsigned)ctas, 256, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A,
+                                                         plan.chunks, plan.max_chunks, plan.partial);
   });
   return cudaGetLastError();
 }
