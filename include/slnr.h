@@ -22,8 +22,13 @@
  *    dimension = number of columns), and 16-byte aligned.
  *  - Index arrays are int32; coordinates are sorted ascending and unique
  *    within each parent (row, slice or fiber); every nnz count is < 2^31.
- *  - Inner dimensions (K, L, M) must each be a power of two in [4, 256];
- *    other values return SLNR_ERR_UNSUPPORTED.
+ *  - Inner dimensions (K, L, M, J) may be any multiple of 4 in [4, 1024];
+ *    other values return SLNR_ERR_UNSUPPORTED.  Powers of two in [4, 256]
+ *    run on kernels specialised for their width (TF32 tensor cores for the
+ *    dense contractions of the fused <SpMM,GEMM>, <SpTTM,SpTTM> and
+ *    <SpMMH,GEMM> with K in {16, 32, 64, 128}, or K = 256 with L <= 64);
+ *    other widths on kernels that take the width at run time, with the same
+ *    schedules.
  *  - Work is enqueued on opts->stream (a cudaStream_t; NULL = the legacy
  *    default stream) and runs asynchronously: the call returns once the
  *    kernels are enqueued.  With opts->validate != 0 the call first checks the

@@ -52,7 +52,10 @@ void timing_end(cudaStream_t s) {
     if (e_ != cudaSuccess) return fail(SLNR_ERR_CUDA, "%s: %s", #expr, cudaGetErrorString(e_)); \
   } while (0)
 
+// Widths the specialised kernels take (powers of two in [4, 256]); any other
+// multiple of 4 up to kWideMax goes to the run-time-width kernels (wide.cu).
 bool pow2_dim(int32_t d) { return d >= 4 && d <= 256 && (d & (d - 1)) == 0; }
+bool all_pow2(int32_t a, int32_t b, int32_t c = 4) { return pow2_dim(a) && pow2_dim(b) && pow2_dim(c); }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -180,7 +183,8 @@ slnr_status check_csf(const slnr_csf3* B, bool need_ptrs) {
 
 slnr_status check_dims(const char* what, int32_t d) {
   if (d <= 0) return fail(SLNR_ERR_SHAPE, "%s = %d must be positive", what, (int)d);
-  if (!pow2_dim(d)) return fail(SLNR_ERR_UNSUPPORTED, "%s = %d: must be a power of two in [4, 256]", what, (int)d);
+  if (!wide_dim(d))
+    return fail(SLNR_ERR_UNSUPPORTED, "%s = %d: must be a multiple of 4 in [4, %d]", what, (int)d, kWideMax);
   return SLNR_OK;
 }
 
@@ -313,6 +317,61 @@ Layout layout_mttkrp_gemm(const slnr_csf3* B, int32_t L, int variant) {
 CsrView csr_view(const slnr_csr* B) { return CsrView{B->nrows, B->ncols, B->nnz, B->pos, B->crd, B->vals}; }
 CsrView fiber_view(const slnr_csf3* B) {
   return CsrView{B->nfibers, B->dim[2], B->nnz, B->pos3, B->crd3, B->vals};
+}
+
+// ---------------------------------------------------------------------------
+// widths outside the specialised kernels (wide.cu): the same schedules with
+// the width chosen at run time
+
+// <SpMM,GEMM> shape (also <SpTTM,SpTTM> over fibers and, with C2, <SpMMH,GEMM>):
+// A = B . (C [.* C2]) . D, C2 NULL or the Hadamard partner of C
+slnr_status wide_spmm_gemm(const CsrView& v, const float* C, const float* C2, int32_t K, const float* D, int32_t L,
+                           float* A, char* ws, const Layout& l, int variant, bool tc, cudaStream_t s) {
+  const SplitPlan sp = split_plan(ws, l);
+  SLNR_LAUNCH("classify", launch_classify(v, sp, s));
+  if (variant == SLNR_FUSED) {
+    SLNR_LAUNCH("w_spmm_chunks", launch_w_spmm(K, v, C, C2, nullptr, sp, s));
+    SLNR_LAUNCH("w_spmm_gemm_tiles", launch_w_spmm_gemm_tiles(K, L, v, C, C2, D, A, s));
+    SLNR_LAUNCH("w_combine", launch_w_combine(K, sp, D, L, A, s));
+  } else {
+    float* T = reinterpret_cast<float*>(ws + l.o_inter);
+    SLNR_LAUNCH("w_spmm", launch_w_spmm(K, v, C, C2, T, sp, s));
+    SLNR_LAUNCH("w_combine", launch_w_combine(K, sp, nullptr, 0, T, s));
+    if (tc)
+      SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(v.nrows, K, L, T, D, A, sp.hdr, s));
+    else
+      SLNR_LAUNCH("w_dense_gemm", launch_w_dense_gemm(v.nrows, K, L, T, D, A, s));
+  }
+  return SLNR_OK;
+}
+
+// MTTKRP (E NULL) or <MTTKRP,GEMM> (times E, L x M); the units are already listed
+slnr_status wide_mttkrp(const slnr_csf3* B, const float* C, const float* D, int32_t L, const float* E, int32_t M,
+                        float* A, char* ws, const Layout& l, const UnitPlan& up, int variant, bool tc,
+                        cudaStream_t s) {
+  if (variant == SLNR_FUSED) {
+    SLNR_LAUNCH("w_mttkrp_units", launch_w_mttkrp_units(L, *B, C, D, nullptr, up, s));
+    SLNR_LAUNCH("w_mttkrp_combine", launch_w_mttkrp_combine(L, *B, up, E, M, A, s));
+    return SLNR_OK;
+  }
+  const CsrView fv = fiber_view(B);
+  const SplitPlan sp = split_plan(ws, l);
+  float* T = reinterpret_cast<float*>(ws + l.o_inter);
+  SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
+  SLNR_LAUNCH("w_spmm", launch_w_spmm(L, fv, D, nullptr, T, sp, s));
+  SLNR_LAUNCH("w_combine", launch_w_combine(L, sp, nullptr, 0, T, s));
+  SLNR_LAUNCH("w_mttkrp_units", launch_w_mttkrp_units(L, *B, C, nullptr, T, up, s));
+  if (E == nullptr) {
+    SLNR_LAUNCH("w_mttkrp_combine", launch_w_mttkrp_combine(L, *B, up, nullptr, 0, A, s));
+    return SLNR_OK;
+  }
+  float* U = reinterpret_cast<float*>(ws + l.o_inter2);
+  SLNR_LAUNCH("w_mttkrp_combine", launch_w_mttkrp_combine(L, *B, up, nullptr, 0, U, s));
+  if (tc)
+    SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->dim[0], L, M, U, E, A, sp.hdr, s));
+  else
+    SLNR_LAUNCH("w_dense_gemm", launch_w_dense_gemm(B->dim[0], L, M, U, E, A, s));
+  return SLNR_OK;
 }
 
 }  // namespace
@@ -472,6 +531,8 @@ slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const f
     SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
     SLNR_LAUNCH("tc_spmm_gemm", launch_tc_spmm_gemm(K, L, v, C, D, A, gp, s));
     SLNR_LAUNCH("combine", launch_combine(L, combine_plan(gp), nullptr, 0, A, s));
+  } else if (!all_pow2(K, L)) {
+    SLNR_CHECK(wide_spmm_gemm(v, C, nullptr, K, D, L, A, ws, l, opts->variant, tc, s));
   } else {
     const SplitPlan sp = split_plan(ws, l);
     SLNR_LAUNCH("classify", launch_classify(v, sp, s));
@@ -514,7 +575,18 @@ slnr_status slnr_sddmm_spmm(const slnr_csr* B, const float* C, const float* D, i
   const CsrView v = csr_view(B);
   const SplitPlan sp = split_plan(ws, l);
   SLNR_LAUNCH("classify", launch_classify(v, sp, s));
-  if (opts->variant == SLNR_FUSED) {
+  if (!all_pow2(L, K)) {
+    if (opts->variant == SLNR_FUSED) {
+      SLNR_LAUNCH("w_sddmm_spmm", launch_w_sddmm_spmm(v, C, D, L, E, K, A, nullptr, sp, s));
+    } else {
+      float* Y = reinterpret_cast<float*>(ws + l.o_inter);
+      SLNR_LAUNCH("w_sddmm", launch_w_sddmm_spmm(v, C, D, L, nullptr, K, nullptr, Y, sp, s));
+      CsrView vy = v;
+      vy.vals = Y;
+      SLNR_LAUNCH("w_spmm", launch_w_spmm(K, vy, E, nullptr, A, sp, s));
+    }
+    SLNR_LAUNCH("w_combine", launch_w_combine(K, sp, nullptr, 0, A, s));
+  } else if (opts->variant == SLNR_FUSED) {
     SLNR_LAUNCH("sddmm_spmm_rows", launch_sddmm_spmm_rows(v, C, D, L, E, K, A, sp, s));
     SLNR_LAUNCH("combine", launch_combine(K, sp, nullptr, 0, A, s));
   } else {
@@ -549,6 +621,10 @@ slnr_status slnr_mttkrp(const slnr_csf3* B, const float* C, const float* D, int3
                    [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
   const UnitPlan up = unit_plan(ws, l);
   SLNR_LAUNCH("csf_units", launch_csf_units(*B, up, s));
+  if (!pow2_dim(L)) {
+    SLNR_CHECK(wide_mttkrp(B, C, D, L, nullptr, 0, A, ws, l, up, opts->variant, false, s));
+    return finish(ws, s, opts->validate != 0);
+  }
   if (opts->variant == SLNR_FUSED) {
     SLNR_LAUNCH("mttkrp_units", launch_mttkrp_units(L, *B, C, D, up, s));
   } else {
@@ -602,6 +678,8 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
     SLNR_LAUNCH("seg_write", launch_seg_write(fv, gp, s));
     SLNR_LAUNCH("tc_spmm_gemm", launch_tc_spmm_gemm(L, M, fv, C, D, A_vals, gp, s));
     SLNR_LAUNCH("combine", launch_combine(M, combine_plan(gp), nullptr, 0, A_vals, s));
+  } else if (!all_pow2(L, M)) {
+    SLNR_CHECK(wide_spmm_gemm(fv, C, nullptr, L, D, M, A_vals, ws, l, opts->variant, tc, s));
   } else {
     const SplitPlan sp = split_plan(ws, l);
     SLNR_LAUNCH("classify", launch_classify(fv, sp, s));
@@ -646,7 +724,25 @@ slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float*
   const CsrView v = csr_view(B);
   const SplitPlan sp = split_plan(ws, l);
   SLNR_LAUNCH("classify", launch_classify(v, sp, s));
-  if (opts->variant == SLNR_FUSED) {
+  if (!all_pow2(K, L, M)) {
+    if (opts->variant == SLNR_FUSED) {
+      SLNR_LAUNCH("w_sddmm_spmm_chunks", launch_w_sddmm_spmm(v, C, D, K, F, L, nullptr, nullptr, sp, s));
+      SLNR_LAUNCH("w_sddmm_spmm_gemm_tiles", launch_w_sddmm_spmm_gemm_tiles(v, C, D, K, F, L, W, M, A, s));
+      SLNR_LAUNCH("w_combine", launch_w_combine(L, sp, W, M, A, s));
+    } else {
+      float* Y = reinterpret_cast<float*>(ws + l.o_inter);
+      float* T = reinterpret_cast<float*>(ws + l.o_inter2);
+      SLNR_LAUNCH("w_sddmm", launch_w_sddmm_spmm(v, C, D, K, nullptr, L, nullptr, Y, sp, s));
+      CsrView vy = v;
+      vy.vals = Y;
+      SLNR_LAUNCH("w_spmm", launch_w_spmm(L, vy, F, nullptr, T, sp, s));
+      SLNR_LAUNCH("w_combine", launch_w_combine(L, sp, nullptr, 0, T, s));
+      if (use_tc(opts, L, M))
+        SLNR_LAUNCH("tc_dense_gemm", launch_tc_dense_gemm(B->nrows, L, M, T, W, A, sp.hdr, s));
+      else
+        SLNR_LAUNCH("w_dense_gemm", launch_w_dense_gemm(B->nrows, L, M, T, W, A, s));
+    }
+  } else if (opts->variant == SLNR_FUSED) {
     // heavy rows: partial T rows (width L), then their fixed-order sum times W
     SLNR_LAUNCH("sddmm_spmm_chunks", launch_sddmm_spmm_chunks(v, C, D, K, F, L, sp, s));
     SLNR_LAUNCH("sddmm_spmm_gemm_tiles", launch_sddmm_spmm_gemm_tiles(v, C, D, K, F, L, W, M, A, s));
@@ -690,7 +786,9 @@ slnr_status slnr_mttkrp_gemm(const slnr_csf3* B, const float* C, const float* D,
                    [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
   const UnitPlan up = unit_plan(ws, l);
   SLNR_LAUNCH("csf_units", launch_csf_units(*B, up, s));
-  if (opts->variant == SLNR_FUSED) {
+  if (!all_pow2(L, M)) {
+    SLNR_CHECK(wide_mttkrp(B, C, D, L, E, M, A, ws, l, up, opts->variant, use_tc(opts, L, M), s));
+  } else if (opts->variant == SLNR_FUSED) {
     SLNR_LAUNCH("mttkrp_units", launch_mttkrp_units(L, *B, C, D, up, s));
     SLNR_LAUNCH("mttkrp_combine", launch_mttkrp_combine(L, *B, up, E, M, A, s));
   } else {
@@ -740,6 +838,8 @@ slnr_status slnr_spmmh_gemm(const slnr_csr* B, const float* C, const float* D, i
     SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
     SLNR_LAUNCH("tc_spmmh_gemm", launch_tc_spmm_gemm(J, L, v, C, E, A, gp, s, D));
     SLNR_LAUNCH("combine", launch_combine(L, combine_plan(gp), nullptr, 0, A, s));
+  } else if (!all_pow2(J, L)) {
+    SLNR_CHECK(wide_spmm_gemm(v, C, D, J, E, L, A, ws, l, opts->variant, tc, s));
   } else {
     const SplitPlan sp = split_plan(ws, l);
     SLNR_LAUNCH("classify", launch_classify(v, sp, s));

@@ -126,6 +126,32 @@ cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T
 cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M,
                                   float* A, cudaStream_t s);
 
+// wide.cu -- any inner width that is a multiple of 4 up to kWideMax, chosen at
+// run time (the kernels above take powers of two in [4, 256])
+constexpr int kWideMax = 1024;
+bool wide_dim(int d);
+// out = B . X (width W; with X2, the gathered row is X .* X2): light rows to
+// out, heavy rows' chunks to plan.partial (then launch_w_combine)
+cudaError_t launch_w_spmm(int W, const CsrView& B, const float* X, const float* X2, float* out,
+                          const SplitPlan& plan, cudaStream_t s);
+// heavy rows: out[row,:] = sum of the row's partials (width W), times D (W x L) when D is not NULL
+cudaError_t launch_w_combine(int W, const SplitPlan& plan, const float* D, int L, float* out, cudaStream_t s);
+// fused B . C . D over light rows (T tile on chip); with C2, the gathered row is C .* C2
+cudaError_t launch_w_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* C, const float* C2,
+                                     const float* D, float* A, cudaStream_t s);
+cudaError_t launch_w_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A, cudaStream_t s);
+// fused <SDDMM,SpMM> (C nrows x Kd, D ncols x Kd, E ncols x Ko): light rows to A,
+// heavy rows' chunks to plan.partial; with Y not NULL, only the sampled products Y[p]
+cudaError_t launch_w_sddmm_spmm(const CsrView& B, const float* C, const float* D, int Kd, const float* E, int Ko,
+                                float* A, float* Y, const SplitPlan& plan, cudaStream_t s);
+cudaError_t launch_w_sddmm_spmm_gemm_tiles(const CsrView& B, const float* C, const float* D, int K, const float* F,
+                                           int L, const float* W, int M, float* A, cudaStream_t s);
+// MTTKRP unit partials: fused (T == NULL) or from the per-fiber T (unfused)
+cudaError_t launch_w_mttkrp_units(int L, const slnr_csf3& B, const float* C, const float* D, const float* T,
+                                  const UnitPlan& plan, cudaStream_t s);
+cudaError_t launch_w_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M, float* A,
+                                    cudaStream_t s);
+
 }  // namespace slnr
 
 // Runs `body` with a compile-time constant WCONST equal to the runtime width

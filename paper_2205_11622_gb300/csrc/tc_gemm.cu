@@ -268,6 +268,12 @@ __host__ __device__ constexpr int tc_nbuf(int K, int L) {
                    : 1;
 }
 
+// Tensor memory columns a CTA allocates: its NBUF accumulators (L columns
+// each), at least the 32 columns an allocation takes.
+__host__ __device__ constexpr uint32_t tc_tmem_cols(int K, int L) {
+  return tc_nbuf(K, L) * L < 32 ? 32u : (uint32_t)(tc_nbuf(K, L) * L);
+}
+
 // Epilogue staging: each of the four epilogue warps stages its 32 rows, one
 // column chunk of min(L, 32) values at a time, in shared memory with a row
 // pitch padded by 16 bytes (the warp's 16-byte stores of 32 different rows
@@ -307,7 +313,7 @@ __device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("pre
 // least 8 items).
 template <int K>
 struct ProdLayout {
-  static constexpr int VPL = 4;
+  static constexpr int VPL = K > 128 ? 8 : 4;  // a group is at most a warp
   static constexpr int GS = K / VPL;
   static constexpr int G = 32 / GS;
   static constexpr int R = GS < kBatch ? GS : kBatch;
@@ -420,7 +426,7 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
                                            const int32_t* __restrict__ crd, const float* __restrict__ vals,
                                            const float* __restrict__ X, const float* __restrict__ X2, int col,
                                            Place& pl) {
-  constexpr int B0 = H ? kBatch / 2 : kBatch;  // two loads per nonzero with H
+  constexpr int B0 = (H ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (H ? kBatch / 2 : kBatch) * 4 / VPL : 1;  // the same registers for any row width and with H
   constexpr int B = B0 < GS ? B0 : GS;
   static_assert(GS % B == 0, "batches tile a chunk");
   constexpr int LPR = K * 4 / 128 > 0 ? K * 4 / 128 : 1;  // 128-byte lines per gathered row
@@ -627,13 +633,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
               const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ D,
               float* __restrict__ A, float* __restrict__ partial, long long wait_cycles) {
-  static_assert(K == 16 || K == 32 || K == 64 || K == 128, "K must be 16, 32, 64 or 128");
+  static_assert(K == 16 || K == 32 || K == 64 || K == 128 || K == 256, "K must be 16, 32, 64, 128 or 256");
   static_assert(L % 16 == 0 && L >= 16 && L <= 256, "L must be a multiple of 16 in [16, 256]");
   constexpr int KT = tc_kt(K);  // tile columns (K, or 32 with zero padding)
   using PL = ProdLayout<K>;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
-  constexpr uint32_t NCOLS = NBUF * L;  // TMEM columns: NBUF fp32 accumulators
+  // TMEM columns: NBUF fp32 accumulators of L columns; an allocation is a
+  // power of two of at least 32 columns
+  constexpr uint32_t NCOLS = tc_tmem_cols(K, L);
+  static_assert(NCOLS >= (uint32_t)(NBUF * L) && NCOLS >= 32 && (NCOLS & (NCOLS - 1)) == 0 && NCOLS <= 512,
+                "tensor memory allocation");
   constexpr int TBYTES = kTcRows * KT * 4;
   constexpr int CPT = kTcRows / PL::IPC;  // claims per item tile
   static_assert(NBUF <= kMaxBuf, "buffers");
@@ -779,7 +789,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // The list is sorted by length class, longest first: no item after
         // item0 has more nonzeros than item0's class bound, so item0 picks
         // the wave shape for the group's R items.
-        constexpr int BW = H ? kBatch / 2 : kBatch;  // rows in flight per group (two loads each with H)
+        // rows in flight per group: fewer with two loads each (H) or 8 columns per lane
+        constexpr int BW = (H ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (H ? kBatch / 2 : kBatch) * 4 / VPL : 1;
         constexpr int W1 = R < BW ? R : BW;
         constexpr int W2 = R < BW / 2 ? R : (BW / 2 > 1 ? BW / 2 : 1);
         constexpr int W4 = R < BW / 4 ? R : (BW / 4 > 1 ? BW / 4 : 1);
@@ -925,7 +936,7 @@ cudaError_t tc_setup(TcLaunch* out) {
   size_t smem = tc_smem_bytes(K, L);
   // no more resident CTAs per SM than tensor memory (512 columns) holds
   // accumulators for: a CTA waiting in tcgen05.alloc would only idle
-  const int max_ctas = 512 / (tc_nbuf(K, L) * L);
+  const int max_ctas = 512 / (int)tc_tmem_cols(K, L);
   const size_t floor_bytes = (size_t)sm_smem / (size_t)(max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
   if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE, PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
@@ -969,6 +980,7 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
   SLNR_TC_CASE(32, 16) SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
   SLNR_TC_CASE(64, 16) SLNR_TC_CASE(64, 32) SLNR_TC_CASE(64, 64) SLNR_TC_CASE(64, 128) SLNR_TC_CASE(64, 256)
   SLNR_TC_CASE(128, 16) SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128) SLNR_TC_CASE(128, 256)
+  SLNR_TC_CASE(256, 16) SLNR_TC_CASE(256, 32) SLNR_TC_CASE(256, 64)
 #undef SLNR_TC_CASE
   return cudaErrorInvalidValue;
 }
@@ -989,7 +1001,8 @@ size_t l2_bytes() {
 }  // namespace
 
 bool tc_supported(int K, int L) {
-  return (K == 16 || K == 32 || K == 64 || K == 128) && (L == 16 || L == 32 || L == 64 || L == 128 || L == 256) &&
+  return (K == 16 || K == 32 || K == 64 || K == 128 || (K == 256 && L <= 64)) &&
+         (L == 16 || L == 32 || L == 64 || L == 128 || L == 256) &&
          tc_smem_bytes(K, L) <= (size_t)220 * 1024;
 }
 

@@ -64,10 +64,12 @@ def test_workspace_query_and_argument_errors(lib):
     ou = _opts(variant=1)
     assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 32, 64, ctypes.byref(ou), ctypes.byref(n)) == 0
     assert n.value >= fused + 1000 * 32 * 4          # the materialised T
-    # unsupported inner dimension (not a power of two in [4, 256])
-    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 48, 64, ctypes.byref(o), ctypes.byref(n)) == 5
-    assert "power of two" in slnr.last_error()
-    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 32, 512, ctypes.byref(o), ctypes.byref(n)) == 5
+    # inner dimensions: any multiple of 4 in [4, 1024]; others are unsupported
+    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 48, 64, ctypes.byref(o), ctypes.byref(n)) == 0
+    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 32, 512, ctypes.byref(o), ctypes.byref(n)) == 0
+    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 50, 64, ctypes.byref(o), ctypes.byref(n)) == 5
+    assert "multiple of 4" in slnr.last_error()
+    assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 32, 1028, ctypes.byref(o), ctypes.byref(n)) == 5
     assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 0, 64, ctypes.byref(o), ctypes.byref(n)) == 2
     # bad options
     assert lib.slnr_spmm_gemm_workspace(ctypes.byref(B), 32, 64, None, ctypes.byref(n)) == 1
