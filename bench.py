@@ -106,9 +106,13 @@ def useful_flops(w) -> int:
     return int(row_flops(w).sum())
 
 
-def min_bytes(w) -> int:
+def min_bytes(w, referenced_only: bool = True) -> int:
     """Bytes an ideal evaluation moves: sparse structure and values once, each
-    dense operand row that is actually referenced once, every output once."""
+    dense operand row that is actually referenced once (every row of every
+    dense input with referenced_only=False, the count that names every dense
+    input once), every output once."""
+    if not referenced_only:
+        return min_bytes_all_rows(w)
     d, B = w.dims, w.B
     if w.op == "spmm_gemm":
         K, L = d["K"], d["L"]
@@ -138,6 +142,39 @@ def min_bytes(w) -> int:
         out_index = 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers
         return structure + 4 * L * _distinct(B.crd3) + 4 * L * M + 4 * B.nfibers * M + out_index
     raise ValueError(w.op)
+
+
+def min_bytes_all_rows(w) -> int:
+    """min_bytes with every row of every dense input read once."""
+    B = w.B
+    dense = sum(int(v.size) * 4 for v in w.dense.values())
+    if w.op in CSR_OPS:
+        sparse = 4 * (B.nrows + 1) + 8 * B.nnz
+    else:
+        sparse = 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers + 4 * (B.nfibers + 1) + 8 * B.nnz
+    d = w.dims
+    if w.op in CSR_OPS:
+        width = {"spmm_gemm": "L", "sddmm_spmm": "K", "sddmm_spmm_gemm": "M", "spmmh_gemm": "L"}[w.op]
+        out = 4 * B.nrows * d[width]
+    elif w.op == "spttm_ttm":
+        out = 4 * B.nfibers * d["M"] + 8 + 4 * B.nslices + 4 * (B.nslices + 1) + 4 * B.nfibers
+    else:
+        out = 4 * B.dims[0] * (d["M"] if w.op == "mttkrp_gemm" else d["L"])
+    return sparse + dense + out
+
+
+def consumer_flops(w) -> int:
+    """Flops of the dense consumer contraction (the tensor-core part where it
+    runs on TF32): 2 K L per non-empty row of <SpMM,GEMM>, 2 L M per fiber of
+    <SpTTM,SpTTM>, 2 J L per non-empty row of <SpMMH,GEMM>; 0 otherwise."""
+    d = w.dims
+    if w.op in ("spmm_gemm", "spmmh_gemm"):
+        n = np.diff(w.B.pos)
+        k = d["K"] if w.op == "spmm_gemm" else d["J"]
+        return int(2 * np.count_nonzero(n) * k * d["L"])
+    if w.op == "spttm_ttm":
+        return int(2 * w.B.nfibers * d["L"] * d["M"])
+    return 0
 
 
 def kernel_source_hash() -> str:
@@ -456,20 +493,41 @@ def main():
     per_expression = {}
     for i, w in enumerate(ws):
         kms = {k: round(v / args.steps, 4) for k, v in kern_ms[i].items()}
+        all_rows = min_bytes_all_rows(w)
         per_expression[w.name] = {
             "ms": round(mean_ms[i], 4), "gflops": round(flops[i] / (mean_ms[i] / 1e3) / 1e9, 2),
             "min_bytes": mbytes[i], "gbs": round(mbytes[i] / (mean_ms[i] / 1e3) / 1e9, 1),
             "hbm_frac": round(mbytes[i] / (mean_ms[i] / 1e3) / 1e9 / peak, 4),
-            "kernels_ms": kms, "useful_flops": flops[i]}
+            "min_bytes_all_rows": all_rows, "hbm_frac_all_rows": round(all_rows / (mean_ms[i] / 1e3) / 1e9 / peak, 4),
+            "kernels_ms": kms, "useful_flops": flops[i], "in_headline": True}
+    # config 1 (the small <SpMM,GEMM>, launch-bound): timed the same way, reported beside the step
+    small = config1_latency(torch, slnr, dev, args, allow_tf32, flush_buf, stream)
+    per_expression[small["name"]] = small["entry"]
+    # the dominant call and, inside it, its dominant kernel (the timing hook's per-launch events)
     dom = int(np.argmax(mean_ms))
     dw = ws[dom]
-    achieved = mbytes[dom] / (mean_ms[dom] / 1e3) / 1e9
+    kname = max(kern_ms[dom], key=kern_ms[dom].get)
+    k_ms = kern_ms[dom][kname] / args.steps
+    achieved = mbytes[dom] / (k_ms / 1e3) / 1e9
+    all_rows = min_bytes_all_rows(dw)
     traffic = ncu_traffic(dw.name)
+    pk = slnr.peaks(stream) if rank == 0 else {}
+    cflops = consumer_flops(dw)
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "traffic": traffic,
-                "kernel": f"{dw.name}: the fused call (launches {', '.join(kern_ms[dom].keys())}), "
-                          f"{mbytes[dom]} algorithmic bytes per call",
-                "peak_kind": f"{peak_kind} HBM copy bandwidth"}
+                "kernel": f"{kname} of {dw.name} ({k_ms:.4f} ms per launch); achieved = the call's "
+                          f"{mbytes[dom]} algorithmic bytes (each referenced dense row once) per launch",
+                "peak_kind": f"{peak_kind} HBM copy bandwidth",
+                "frac_call": round(mbytes[dom] / (mean_ms[dom] / 1e3) / 1e9 / peak, 4),
+                "min_bytes_all_rows": all_rows,
+                "frac_all_rows": round(all_rows / (k_ms / 1e3) / 1e9 / peak, 4),
+                "compute": {"unit": "TFLOP/s", "tf32_peak_measured": round(pk.get("tf32_tflops", 0.0), 1),
+                            "ffma_peak_measured": round(pk.get("ffma_tflops", 0.0), 1),
+                            "tf32_achieved": round(cflops / (k_ms / 1e3) / 1e12, 2),
+                            "tf32_frac": round(cflops / (k_ms / 1e3) / 1e12 / pk["tf32_tflops"], 4)
+                            if pk.get("tf32_tflops") else None,
+                            "note": "the dense consumer contraction of the dominant kernel (2 K L per non-empty "
+                                    "row) against this library's own tcgen05 kind::tf32 peak kernel"}}
 
     cpu = None
     if rank == 0 and world == 1 and not args.skip_cpu:
@@ -499,7 +557,7 @@ def main():
     return 0
 
 
-SWEEP_DIMS = (16, 32, 64, 128, 256)
+SWEEP_DIMS = (16, 32, 64, 128, 256, 512)
 
 
 def run_sweep(args, rank, world, local):
@@ -567,6 +625,34 @@ def run_sweep(args, rank, world, local):
     if rank == 0:
         print(json.dumps(line))
     return 0
+
+
+def config1_latency(torch, slnr, dev, args, allow_tf32, flush_buf, stream):
+    """Config 1 (<SpMM,GEMM> on a 1024^2 matrix with 10 uniform nonzeros per
+    row, K = L = 32): far too small for a bandwidth roofline (it fits in L2),
+    so its latency is reported beside the step, not in the headline value.
+    Same protocol: warm-up, L2 flushed before each call, CUDA events."""
+    w = wl.full(0)
+    B = slnr.DeviceCSR.from_host(w.B, dev)
+    dense = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dev) for k, v in w.dense.items()}
+    ws = slnr.Workspace(device=dev)
+    out = slnr.run(w.op, B, dense, variant=args.variant, allow_tf32=allow_tf32, workspace=ws)
+    ts = []
+    for it in range(args.warmup + args.steps):
+        flush_buf.fill_(it & 0xFF)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        slnr.run(w.op, B, dense, out=out, variant=args.variant, allow_tf32=allow_tf32, workspace=ws)
+        b.record(stream)
+        b.synchronize()
+        if it >= args.warmup:
+            ts.append(a.elapsed_time(b))
+    kt = slnr.timing_read()
+    ms = statistics.mean(ts)
+    return {"name": w.name, "entry": {
+        "ms": round(ms, 4), "gflops": round(useful_flops(w) / (ms / 1e3) / 1e9, 2), "min_bytes": min_bytes(w),
+        "kernels_ms": {k: round(v, 4) for k, v in kt}, "useful_flops": useful_flops(w), "in_headline": False,
+        "note": "config 1, latency-bound (fits in L2): timed beside the step, not part of value"}}
 
 
 def measure_e2e(torch, slnr, ws, dev_inputs, outs, call, stream, steps, total_flops, world, pg, dev):

@@ -210,16 +210,18 @@ slnr_status slnr_spmmh_gemm(const slnr_csr *B, const float *C, const float *D, i
 
 /* ---- <SDDMM,SpMM> without a caller workspace ----------------------------
  * The paper has no counterpart to this entry point; it serves callers that
- * cannot allocate device memory (code inside a CUDA graph being captured, a
- * real-time or signal-safe path that must not enter an allocator, or a host
- * runtime that owns all device memory).  It runs the fused variant of
+ * cannot allocate device memory (a real-time or signal-safe path that must
+ * not enter an allocator, which can block or take locks, or a host runtime
+ * that owns all device memory and hands none to the libraries it hosts).  It runs the fused variant of
  * slnr_sddmm_spmm with the same arguments and results, but its scratch is a
  * 16 MiB array inside the library's device code: every GPU that loads the
  * library holds those 16 MiB until the process exits, and the call allocates
  * nothing.  Sizes whose scratch would exceed 16 MiB (about 7 million nonzeros
  * at K = 64) return SLNR_ERR_UNSUPPORTED.  The first call on each device
  * looks up the array's device address (cudaGetSymbolAddress) with that device
- * current; make that first call before any stream capture begins.  All calls
+ * current and keeps it; make that first call before any stream capture
+ * begins.  A device reset (cudaDeviceReset) leaves the kept address stale:
+ * do not call this entry point on a device after resetting it.  All calls
  * share the one array: the call clears what must start at zero itself, and
  * calls whose work overlaps on the GPU (other streams, other host threads)
  * race on it.  Runs on `stream` (a cudaStream_t, NULL = legacy default), with
@@ -251,6 +253,17 @@ slnr_status slnr_timing_get(int32_t i, const char **name, float *ms);
  * the timeout path; a limit shorter than the work makes correct calls fail.
  * Returns SLNR_ERR_SHAPE for cycles < 0. */
 slnr_status slnr_set_wait_limit(int64_t cycles);
+
+/* ---- compute peaks --------------------------------------------------------
+ * The GPU's FP32 FFMA rate (CUDA cores) and TF32 rate (tcgen05 tensor cores,
+ * kind::tf32, M = 128, N = 256), each measured by a kernel of this library
+ * (a second, timed launch after a first one), in TFLOP/s.  They are the
+ * compute denominators of the roofline the benchmark reports; neither is
+ * part of any expression.  Runs on `stream` (NULL = legacy default) and
+ * waits for it; allocates nothing.  slnr_peak_tf32 returns SLNR_ERR_TIMEOUT
+ * if its bounded wait for the MMAs gave up. */
+slnr_status slnr_peak_ffma(void *stream, double *tflops);
+slnr_status slnr_peak_tf32(void *stream, double *tflops);
 
 /* ---- diagnostics ------------------------------------------------------- */
 const char *slnr_status_string(slnr_status status);

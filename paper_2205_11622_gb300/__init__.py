@@ -72,6 +72,8 @@ SIGNATURES = {
     "slnr_spmmh_gemm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_sddmm_spmm_noalloc": ([_CSR, _P, _P, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "slnr_set_wait_limit": ([ctypes.c_int64], ctypes.c_int),
+    "slnr_peak_ffma": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+    "slnr_peak_tf32": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
     "slnr_timing_get": ([_I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
@@ -117,6 +119,18 @@ def _check(status: int, where: str):
 def timing_enable(on: bool = True):
     """Record CUDA events between the library's launches on this thread (slnr_timing_enable)."""
     _check(lib().slnr_timing_enable(int(bool(on))), "slnr_timing_enable")
+
+
+def peaks(stream=None):
+    """{"ffma_tflops", "tf32_tflops"}: the compute peaks measured by the library's own kernels."""
+    torch = _torch()
+    s = ctypes.c_void_p((stream or torch.cuda.current_stream()).cuda_stream)
+    out = {}
+    for key, fn in (("ffma_tflops", "slnr_peak_ffma"), ("tf32_tflops", "slnr_peak_tf32")):
+        v = ctypes.c_double(0.0)
+        _check(getattr(lib(), fn)(s, ctypes.byref(v)), fn)
+        out[key] = v.value
+    return out
 
 
 def timing_read():

@@ -402,6 +402,20 @@ const char* slnr_last_error(void) { return g_last_error; }
 
 const char* slnr_version(void) { return "slnr 0.2.0 (sm_103a)"; }
 
+slnr_status slnr_peak_ffma(void* stream, double* tflops) {
+  if (!tflops) return fail(SLNR_ERR_NULL, "tflops is NULL");
+  SLNR_CUDA(peak_ffma(static_cast<cudaStream_t>(stream), tflops));
+  return SLNR_OK;
+}
+
+slnr_status slnr_peak_tf32(void* stream, double* tflops) {
+  if (!tflops) return fail(SLNR_ERR_NULL, "tflops is NULL");
+  const cudaError_t e = peak_tf32(static_cast<cudaStream_t>(stream), tflops);
+  if (e == cudaErrorLaunchTimeout) return fail(SLNR_ERR_TIMEOUT, "the TF32 peak kernel's wait gave up");
+  SLNR_CUDA(e);
+  return SLNR_OK;
+}
+
 slnr_status slnr_set_wait_limit(int64_t cycles) {
   if (cycles < 0) return fail(SLNR_ERR_SHAPE, "wait limit must be >= 0");
   g_wait_limit = cycles;

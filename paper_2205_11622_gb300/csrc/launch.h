@@ -152,6 +152,10 @@ cudaError_t launch_w_mttkrp_units(int L, const slnr_csf3& B, const float* C, con
 cudaError_t launch_w_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M, float* A,
                                     cudaStream_t s);
 
+// peaks.cu -- compute peaks measured by the library's own kernels (TFLOP/s)
+cudaError_t peak_ffma(cudaStream_t s, double* tflops);
+cudaError_t peak_tf32(cudaStream_t s, double* tflops);
+
 }  // namespace slnr
 
 // Runs `body` with a compile-time constant WCONST equal to the runtime width

@@ -1,10 +1,10 @@
 // slnr_sddmm_spmm_noalloc: the fused <SDDMM,SpMM> call for callers that
 // cannot allocate device memory.
 //
-// Some callers may not call cudaMalloc at all: code running inside a CUDA
-// graph that is being captured, a real-time or signal-safe path that must
-// not enter the allocator, or an embedding runtime that owns all device
-// memory and hands out none.  This entry point needs no caller workspace:
+// Some callers may not call cudaMalloc at all: a real-time or signal-safe
+// path that must not enter the allocator (which can block or take locks), or
+// an embedding runtime that owns all device memory and hands out none to the
+// libraries it hosts.  This entry point needs no caller workspace:
 // its scratch is the file-scope array below, which the CUDA runtime creates
 // with the module, so every GPU that loads this library holds
 // kNoAllocScratchBytes of device memory until the process exits.
@@ -13,7 +13,9 @@
 // code it names a host-side stand-in), so the first call on each device looks
 // up the array's device address with cudaGetSymbolAddress, with that device
 // current, and caches it.  The first call on a device should therefore be
-// made before any stream capture begins.  Every call shares the one array,
+// made before any stream capture begins.  The cache outlives a device reset
+// (cudaDeviceReset), after which the address is stale: a process that
+// resets a device must not call this entry point on it again.  Every call shares the one array,
 // which keeps the last call's contents: the call clears the part that must
 // start at zero (the header of counters) itself, and calls whose work
 // overlaps on the GPU (different streams, or different host threads on one

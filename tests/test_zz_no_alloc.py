@@ -1,13 +1,16 @@
 """slnr_sddmm_spmm_noalloc against slnr_sddmm_spmm, through the C ABI (GPU).
 
 The no-allocation entry point is for callers that cannot allocate device
-memory (inside a CUDA graph capture, on a real-time path, or under a runtime
+memory (a real-time path that must not enter an allocator, or a host runtime
 that owns all device memory): it takes no workspace and uses a fixed 16 MiB
-scratch array inside the library.  Two calls in a row, on different sizes,
-must each agree with the workspace-taking entry point within the fp32
-tolerance of the other parity tests; sizes beyond the scratch are rejected
-with an explanatory error.  This file is named to run last, and it also
-passes on its own in a fresh process.
+scratch array inside the library.  Calls in a row, on different sizes, must
+each agree with the workspace-taking entry point within the fp32 tolerance
+of the other parity tests, including a large call followed by a smaller one
+and a large one again (the shared array keeps the last call's heavy-row
+records, chunks, partial rows and counters) on a graph with rows past the
+heavy-row threshold.  Sizes beyond the scratch are rejected with an
+explanatory error.  This file is named to run last, and it also passes on
+its own in a fresh process.
 """
 import ctypes
 
@@ -60,6 +63,19 @@ def _call_both(slnr, w):
 def test_noalloc_matches_workspace_entry_point_twice(slnr):
     cases = [wl.small(1), wl.sddmm_spmm_rmat(0x51A4 + 41, 2500, 18, 32, 128)]
     for w in cases:
+        ref_ws, got = _call_both(slnr, w)
+        _, ref_abs = oracle.get().run(w)
+        err = P.rel_err(got, ref_ws.astype(np.float64), ref_abs)
+        assert err <= P.TOL_FP32, f"{w.name}: no-alloc differs from slnr_sddmm_spmm by {err:.3e}"
+
+
+def test_noalloc_large_small_large(slnr):
+    # R-MAT hubs: the large graph has rows above the 256-nonzero threshold
+    # (split into chunks whose partial rows live in the scratch array)
+    large = wl.sddmm_spmm_rmat(0x51A4 + 43, 12000, 24, 64, 64)
+    small = wl.sddmm_spmm_rmat(0x51A4 + 44, 900, 6, 16, 32)
+    assert int(np.max(np.diff(large.B.pos))) > 256, "the large case must have heavy rows"
+    for w in (large, small, large):
         ref_ws, got = _call_both(slnr, w)
         _, ref_abs = oracle.get().run(w)
         err = P.rel_err(got, ref_ws.astype(np.float64), ref_abs)
