@@ -603,8 +603,8 @@ def run_sweep(args, rank, world, local):
                     if it >= args.warmup:
                         ts.append(a.elapsed_time(b))
                 res[f"{variant}_ms"] = round(statistics.median(ts), 4)
-            if slnr.device_flags() != 0:
-                raise SystemExit(f"device flags {slnr.device_flags():#x} at K={K}, L={L}")
+                if slnr.device_flags() != 0:
+                    raise SystemExit(f"device flags {slnr.device_flags():#x} at K={K}, L={L}, {variant}")
             res["unfused_over_fused"] = round(res["unfused_ms"] / res["fused_ms"], 3)
             res["fused_gflops"] = round(res["useful_flops"] / res["fused_ms"] / 1e6, 1)
             res["fused_hbm_frac"] = round(res["min_bytes"] / res["fused_ms"] / 1e6 / measured_peaks()[0], 4)

@@ -406,11 +406,10 @@ __device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, in
     }
   const int sl = pl.take(W);
   if (sl < 0) return false;
-#pragma unroll
-  for (int w = 0; w < W; ++w) pl.put(sl + w, x[w * N]);
-  if (gl >= w0 && gl < w0 + W) pl.put_dest(sl + gl - w0, rdst);
-  pl.publish(sl, W);
-  return true;
+  return pl.template place<W>(sl, [&](int w, int slot) {
+    pl.put(slot, x[w * N]);
+    if (gl == w0 + w) pl.put_dest(slot, rdst);
+  });
 }
 
 // The group's R items one after the other, each T row summed in nonzero
@@ -485,7 +484,7 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
       }
     }
     if (rn != r) {  // the item's last chunk: its T row is complete
-      const int sl = pl.take(1);
+      const int sl = pl.take(1);  // one slot: always inside one slot tile
       if (sl < 0) return false;
       pl.put(sl, acc);
       if (gl == r) pl.put_dest(sl, rdst);
@@ -563,38 +562,57 @@ struct Placer {
   unsigned gmask;
   int gbase, gl, col;
   long long wait_cycles;
-  // First of n consecutive slots, once the buffers of their slot tiles are
-  // free (all four epilogue warps have read the destinations of the tiles
-  // NBUF before, so those tiles' MMAs are done); -1 after a timeout.  A range
-  // may span two slot tiles.
+  // First of n consecutive slots, once the buffer of its slot tile is free
+  // (all four epilogue warps have read the destinations of the tile NBUF
+  // before, so its MMAs are done); -1 after a timeout.  The range may run
+  // into the next slot tile: place() fills it tile by tile.
   __device__ __forceinline__ int take(int n) {
     int sl = 0;
     if (gl == 0) sl = atomicAdd(&g_tc.fill, n);
     sl = __shfl_sync(gmask, sl, gbase);
-    const int tl = (sl + n - 1) / kTcRows;
-    if (tl >= NBUF) {
-      const bool ok = epi_wait_timeout(tl - NBUF + 1, wait_cycles);
-      if (__any_sync(gmask, !ok)) {
-        if (gl == 0) atomicOr(&g_tc.fail_flag, 1);
-        return -1;
-      }
+    return wait_tile(sl / kTcRows) ? sl : -1;
+  }
+  // Waits until slot tile t's buffer is free; false after a timeout.
+  __device__ __forceinline__ bool wait_tile(int t) {
+    if (t < NBUF) return true;
+    const bool ok = epi_wait_timeout(t - NBUF + 1, wait_cycles);
+    if (__any_sync(gmask, !ok)) {
+      if (gl == 0) atomicOr(&g_tc.fail_flag, 1);
+      return false;
     }
-    return sl;
+    return true;
+  }
+  // Stores rows 0 .. W-1 into slots sl .. sl + W - 1 (store(w, slot) puts
+  // row w and its destination) and publishes them.  The rows in the first
+  // slot tile are published before waiting for the next tile's buffer: with
+  // one buffer that wait needs the first tile consumed, which needs them.
+  template <int W, typename F>
+  __device__ __forceinline__ bool place(int sl, F&& store) {
+    const int n1 = min(W, kTcRows - sl % kTcRows);
+#pragma unroll
+    for (int w = 0; w < W; ++w)
+      if (w < n1) store(w, sl + w);
+    publish(sl, n1);
+    if (n1 < W) {
+      if (!wait_tile(sl / kTcRows + 1)) return false;
+#pragma unroll
+      for (int w = 0; w < W; ++w)
+        if (w >= n1) store(w, sl + w);
+      publish(sl + n1, W - n1);
+    }
+    return true;
   }
   __device__ __forceinline__ void put(int slot, const float (&acc)[VPL]) {
     store_t_part<VPL>(tc_tiles() + ((slot / kTcRows) % NBUF) * TBYTES, slot % kTcRows, col, acc);
   }
   __device__ __forceinline__ void put_dest(int slot, int2 d) { g_tc.dest[(slot / kTcRows) % NBUF][slot % kTcRows] = d; }
-  // The rows (and destinations) of slots [sl, sl + n) are stored: make them
-  // visible to the tensor cores and count them on their tiles' barriers.
+  // The rows (and destinations) of slots [sl, sl + n), all in one slot tile,
+  // are stored: make them visible to the tensor cores and count them on the
+  // tile's barrier.
   __device__ __forceinline__ void publish(int sl, int n) {
     tc::fence_proxy_async_smem();
     __syncwarp(gmask);
-    if (gl == 0) {
-      const int n1 = min(n, kTcRows - sl % kTcRows);
-      tc::mbar_arrive_n(&g_tc.full_bar[(sl / kTcRows) % NBUF], (uint32_t)n1);
-      if (n > n1) tc::mbar_arrive_n(&g_tc.full_bar[(sl / kTcRows + 1) % NBUF], (uint32_t)(n - n1));
-    }
+    if (gl == 0) tc::mbar_arrive_n(&g_tc.full_bar[(sl / kTcRows) % NBUF], (uint32_t)n);
   }
 };
 
@@ -768,13 +786,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           if (item0 + r < nitems) ldg_vec<VPL>(x[r], X + (int64_t)(item0 + r) * K + col); else zero_vec(x[r]);
         }
         const int sl = pl.take(R);
-        ok = sl >= 0;
-        if (ok) {
-#pragma unroll
-          for (int r = 0; r < R; ++r) pl.put(sl + r, x[r]);
-          if (gl < R) pl.put_dest(sl + gl, make_int2(item0 + gl < nitems ? item0 + gl : -1, -1));
-          pl.publish(sl, R);
-        }
+        ok = sl >= 0 && pl.template place<R>(sl, [&](int r, int slot) {
+          pl.put(slot, x[r]);
+          if (gl == r) pl.put_dest(slot, make_int2(item0 + r < nitems ? item0 + r : -1, -1));
+        });
       } else {
         constexpr bool H = MODE == kSegmentsH;
         // lane gl < R holds the record of the group's item gl

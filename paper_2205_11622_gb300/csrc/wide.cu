@@ -532,9 +532,11 @@ inline unsigned w_grid(int64_t items) {  // a warp per item, grid-stride beyond 
   return (unsigned)(ctas < 1 ? 1 : ctas);
 }
 
+// Opts the kernel in to `bytes` of dynamic shared memory (the default limit
+// counts the kernel's static shared memory too, so set it whenever any is asked).
 template <typename Kern>
 cudaError_t w_smem(Kern k, size_t bytes) {
-  if (bytes <= 48 * 1024) return cudaSuccess;
+  if (bytes == 0) return cudaSuccess;
   return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 

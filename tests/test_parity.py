@@ -260,3 +260,17 @@ def test_tensor_core_path_on_tiny_inputs(slnr, orc, K, L, nrows):
     w = wl.spmm_gemm_uniform(0x51A4 + 13 * K + L + nrows, nrows, 300, 7, K, L, name=f"tiny_{nrows}")
     check(slnr, orc, w, "fused", True)
     check(slnr, orc, w, "unfused", True)
+
+
+@pytest.mark.parametrize("K,L", [(128, 256), (256, 16), (256, 64)])
+@pytest.mark.parametrize("op", ["spmm_gemm", "spttm_ttm"])
+def test_single_buffer_tensor_core_path(slnr, orc, K, L, op):
+    # one T buffer (the tile and D^T fill shared memory): waves of short
+    # items and single long items make slot ranges that run from one slot
+    # tile into the next, over more than 150 tiles; every wait must end
+    # (the device flag stays 0) and the result match the oracle
+    if op == "spmm_gemm":
+        w = wl.spmm_gemm_rmat(0x51A4 + 19 * K + L, 20000, 12, K, L)
+    else:
+        w = wl.spttm_ttm_powerlaw(0x51A4 + 23 * K + L, (200, 200, 900), 100000, 8.0, 900, K, L)
+    check(slnr, orc, w, "fused", True)

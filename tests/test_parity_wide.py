@@ -52,7 +52,7 @@ VARIANTS = [("fused", False), ("fused", True), ("unfused", False), ("unfused", T
 
 @pytest.mark.gpu
 @pytest.mark.parametrize("K,L", [(256, 64), (256, 256), (512, 64), (64, 512), (1024, 16), (256, 32), (12, 100),
-                                 (300, 20), (4, 1024), (100, 4)])
+                                 (300, 20), (4, 1024), (100, 4), (256, 512), (512, 512)])
 @pytest.mark.parametrize("variant,allow_tf32", VARIANTS)
 def test_spmm_gemm_wide(slnr, orc, K, L, variant, allow_tf32):
     # 700 rows of R-MAT degree 10: a few rows above 256 nonzeros (chunks), a ragged last tile
