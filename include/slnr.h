@@ -180,7 +180,8 @@ slnr_status slnr_spttm_ttm(const slnr_csf3 *B, const float *C, int32_t L, const 
  * Fused: Algorithm 1 applied twice.  Per row i, per stored (i,j) the scalar
  * y = B(i,j) C(i,:).D(j,:) is formed and T(i,:) += y F(j,:) at once; the row's
  * vector temporary T(i,:) (length L) stays on chip and A(i,:) = T(i,:).W
- * follows (fp32 FFMA).  Unfused: the sampled product Y (nnz values) and
+ * follows: on TF32 tensor cores with allow_tf32 when K == L in {32, 64, 128}
+ * and M in {32, 64, 128}, else fp32 FFMA.  Unfused: the sampled product Y (nnz values) and
  * T = Y.F (nrows x L) are written to the workspace, then A = T.W (TF32 tensor
  * cores with allow_tf32, where the widths allow). */
 slnr_status slnr_sddmm_spmm_gemm(const slnr_csr *B, const float *C, const float *D, int32_t K, const float *F,

@@ -253,9 +253,17 @@ slnr_status finish(char* ws, cudaStream_t s, bool validate) {
 // The fused tensor-core path takes row segments; everything else splits heavy rows.
 bool use_tc(const slnr_opts* o, int32_t K, int32_t L) { return o->allow_tf32 != 0 && tc_supported(K, L); }
 
+// The fused tensor-core kernel (persistent CTAs, tensor memory, an inspector
+// pass) pays a fixed cost of some tens of microseconds; below this many
+// nonzeros the fused CUDA-core kernels finish first.
+constexpr int64_t kTcFusedMinNnz = int64_t(1) << 14;
+bool use_tc_fused(const slnr_opts* o, int32_t K, int32_t L, int64_t nnz) {
+  return o->variant == SLNR_FUSED && use_tc(o, K, L) && nnz >= kTcFusedMinNnz;
+}
+
 Layout layout_spmm_gemm(const slnr_csr* B, int32_t K, int32_t L, const slnr_opts* o) {
   Layout l;
-  if (o->variant == SLNR_FUSED && use_tc(o, K, L)) {
+  if (use_tc_fused(o, K, L, B->nnz)) {
     l.segs(B->nrows, B->nnz, L);
   } else {
     l.split(B->nrows, B->nnz, K);
@@ -284,7 +292,7 @@ Layout layout_mttkrp(const slnr_csf3* B, int32_t L, int variant) {
 
 Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opts* o) {
   Layout l;
-  if (o->variant == SLNR_FUSED && use_tc(o, L, M)) {
+  if (use_tc_fused(o, L, M, B->nnz)) {
     l.segs(B->nfibers, B->nnz, M);
   } else {
     l.split(B->nfibers, B->nnz, L);
@@ -293,8 +301,19 @@ Layout layout_spttm_ttm(const slnr_csf3* B, int32_t L, int32_t M, const slnr_opt
   return l;
 }
 
-Layout layout_sddmm_spmm_gemm(const slnr_csr* B, int32_t L, int variant) {
+// The fused <SDDMM,SpMM,GEMM> runs on the tensor-core kernel (sampled rows)
+// when TF32 is allowed and the dot product and the temporary have one width.
+bool use_tc_sampled(const slnr_opts* o, int32_t K, int32_t L, int32_t M, int64_t nnz) {
+  return o->variant == SLNR_FUSED && o->allow_tf32 != 0 && tc_sampled_supported(K, L, M) && nnz >= kTcFusedMinNnz;
+}
+
+Layout layout_sddmm_spmm_gemm(const slnr_csr* B, int32_t K, int32_t L, int32_t M, const slnr_opts* o) {
+  const int variant = o->variant;
   Layout l;
+  if (use_tc_sampled(o, K, L, M, B->nnz)) {
+    l.segs(B->nrows, B->nnz, M);
+    return l;
+  }
   l.split(B->nrows, B->nnz, L);
   if (variant == SLNR_UNFUSED) {
     l.inter(sizeof(float) * (size_t)B->nnz);                      // Y
@@ -493,7 +512,7 @@ slnr_status slnr_sddmm_spmm_gemm_workspace(const slnr_csr* B, int32_t K, int32_t
   SLNR_CHECK(check_dims("L", L));
   SLNR_CHECK(check_dims("M", M));
   if (!bytes) return fail(SLNR_ERR_NULL, "bytes is NULL");
-  *bytes = layout_sddmm_spmm_gemm(B, L, opts->variant).total();
+  *bytes = layout_sddmm_spmm_gemm(B, K, L, M, opts).total();
   return SLNR_OK;
 }
 
@@ -539,7 +558,7 @@ slnr_status slnr_spmm_gemm(const slnr_csr* B, const float* C, int32_t K, const f
                    [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
   const CsrView v = csr_view(B);
   const bool tc = use_tc(opts, K, L);
-  if (opts->variant == SLNR_FUSED && tc) {
+  if (use_tc_fused(opts, K, L, B->nnz)) {
     const SegPlan gp = seg_plan(ws, l);
     SLNR_LAUNCH("seg_count", launch_seg_count(v, gp, s));
     SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
@@ -686,7 +705,7 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
   if (B->nfibers == 0) return SLNR_OK;
   const CsrView fv = fiber_view(B);
   const bool tc = use_tc(opts, L, M);
-  if (opts->variant == SLNR_FUSED && tc) {
+  if (use_tc_fused(opts, L, M, B->nnz)) {
     const SegPlan gp = seg_plan(ws, l);
     SLNR_LAUNCH("seg_count", launch_seg_count(fv, gp, s));
     SLNR_LAUNCH("seg_write", launch_seg_write(fv, gp, s));
@@ -728,7 +747,7 @@ slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float*
   SLNR_CHECK(check_dense("F", F));
   SLNR_CHECK(check_dense("W", W));
   SLNR_CHECK(check_dense("A", A));
-  const Layout l = layout_sddmm_spmm_gemm(B, L, opts->variant);
+  const Layout l = layout_sddmm_spmm_gemm(B, K, L, M, opts);
   SLNR_CHECK(check_ws(opts, l.total()));
   if (B->nrows == 0) return SLNR_OK;
   cudaStream_t s = static_cast<cudaStream_t>(opts->stream);
@@ -736,6 +755,16 @@ slnr_status slnr_sddmm_spmm_gemm(const slnr_csr* B, const float* C, const float*
   SLNR_CHECK(begin(ws, s, opts->validate != 0,
                    [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
   const CsrView v = csr_view(B);
+  if (use_tc_sampled(opts, K, L, M, B->nnz)) {
+    // T(i,:) built on chip by the producers, T.W on the TF32 tensor cores;
+    // heavy rows' chunk rows of A are summed by the combine
+    const SegPlan gp = seg_plan(ws, l);
+    SLNR_LAUNCH("seg_count", launch_seg_count(v, gp, s));
+    SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));
+    SLNR_LAUNCH("tc_sddmm_spmm_gemm", launch_tc_sddmm_spmm_gemm(v, C, D, F, L, W, M, A, gp, s));
+    SLNR_LAUNCH("combine", launch_combine(M, combine_plan(gp), nullptr, 0, A, s));
+    return finish(ws, s, opts->validate != 0);
+  }
   const SplitPlan sp = split_plan(ws, l);
   SLNR_LAUNCH("classify", launch_classify(v, sp, s));
   if (!all_pow2(K, L, M)) {
@@ -845,8 +874,9 @@ slnr_status slnr_spmmh_gemm(const slnr_csr* B, const float* C, const float* D, i
                    [&](WsHeader* h) { return launch_validate_csr(*B, h, s); }));
   const CsrView v = csr_view(B);
   const bool tc = use_tc(opts, J, L);
+  const bool tc_fused = use_tc_fused(opts, J, L, B->nnz);
   // the gathered row of column k is C(k,:) .* D(k,:); E is the consumer matrix
-  if (opts->variant == SLNR_FUSED && tc) {
+  if (tc_fused) {
     const SegPlan gp = seg_plan(ws, l);
     SLNR_LAUNCH("seg_count", launch_seg_count(v, gp, s));
     SLNR_LAUNCH("seg_write", launch_seg_write(v, gp, s));

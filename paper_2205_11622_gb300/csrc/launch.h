@@ -100,6 +100,11 @@ cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, 
                                 const SegPlan& plan, cudaStream_t s, const float* C2 = nullptr);
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s);
+// fused <SDDMM,SpMM,GEMM> on the tensor-core kernel: C nrows x K, D ncols x K,
+// F ncols x L, W L x M, with K == L (the dot product and the temporary share the lane layout)
+bool tc_sampled_supported(int K, int L, int M);
+cudaError_t launch_tc_sddmm_spmm_gemm(const CsrView& B, const float* C, const float* D, const float* F, int L,
+                                      const float* W, int M, float* A, const SegPlan& plan, cudaStream_t s);
 
 // sddmm.cu
 // fused <SDDMM,SpMM>: the heavy rows' chunks (partials) and the light rows in

@@ -251,7 +251,9 @@ __device__ __forceinline__ int mbar_wait_or_end(uint64_t* bar, uint32_t parity, 
 
 // kSegments: gathered row segments; kSegmentsH: the same with Hadamard rows
 // X[k,:] .* X2[k,:] (<SpMMH,GEMM>); kDense: rows of a materialised T.
-enum TcMode { kSegments = 0, kDense = 1, kSegmentsH = 2 };
+// kSampled (<SDDMM,SpMM,GEMM>): the row of stored (i,j) is F(j,:) scaled by
+// the sampled product B(i,j) <C(i,:), D(j,:)>.
+enum TcMode { kSegments = 0, kDense = 1, kSegmentsH = 2, kSampled = 3 };
 
 // Columns of the T tile and of D^T: K, padded to one 128-byte swizzle atom
 // (32 tf32 values) when K = 16; the padding columns hold zeros.
@@ -301,6 +303,41 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 #define SLNR_TC_BATCH 4  // gathered rows a lane group keeps in flight (one batch; half with Hadamard rows)
 #endif
 constexpr int kBatch = SLNR_TC_BATCH;
+
+#ifndef SLNR_TC_STREAM_HINT
+#define SLNR_TC_STREAM_HINT 1  // 1: streamed loads and stores carry an L2 evict-first hint
+#endif
+
+// Loads and stores of data each call streams through once (coordinates,
+// values, segment records, output rows).  With SLNR_TC_STREAM_HINT they are
+// marked evict-first in L2, so that they make room before the gathered rows,
+// which are read again.
+__device__ __forceinline__ uint64_t stream_policy() {
+  uint64_t pol = 0;
+  if (SLNR_TC_STREAM_HINT) asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ int ld_stream(const int32_t* p, uint64_t pol) {
+  if (!SLNR_TC_STREAM_HINT) return __ldg(p);
+  int v;
+  asm volatile("ld.global.nc.L2::cache_hint.b32 %0, [%1], %2;" : "=r"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ float ld_stream(const float* p, uint64_t pol) {
+  if (!SLNR_TC_STREAM_HINT) return __ldg(p);
+  float v;
+  asm volatile("ld.global.nc.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ void st_stream(float* p, float4 x, uint64_t pol) {
+  if (!SLNR_TC_STREAM_HINT) {
+    *reinterpret_cast<float4*>(p) = x;
+    return;
+  }
+  asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(x.x), "f"(x.y), "f"(x.z),
+               "f"(x.w), "l"(pol)
+               : "memory");
+}
 
 // L2 prefetch of the 128-byte line holding p (no register, nothing to wait for).
 __device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
@@ -385,8 +422,9 @@ __device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, in
     const int t = gl + h * GS, w = t / N < W ? t / N : W - 1, s = t % N;
     const int p0 = __shfl_sync(gmask, rp0, gbase + w0 + w), p1 = __shfl_sync(gmask, rp1, gbase + w0 + w);
     const bool ok = t < S && p0 + s < p1;
-    mc[h] = ok ? __ldg(crd + p0 + s) : -1;
-    mv[h] = ok ? __ldg(vals + p0 + s) : 0.f;
+    const uint64_t pol = stream_policy();
+    mc[h] = ok ? ld_stream(crd + p0 + s, pol) : -1;
+    mv[h] = ok ? ld_stream(vals + p0 + s, pol) : 0.f;
   }
   float x[S][VPL];
 #pragma unroll
@@ -420,12 +458,16 @@ __device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, in
 // is gathered.  With PF the chunk after that is loaded too, and the rows of
 // the next chunk are prefetched into L2 (one lane per row,
 // prefetch.global.L2, no register held) while this chunk is gathered.
-template <int K, int VPL, int GS, int R, bool PF, bool H, typename Place>
+// With S (sampled rows, <SDDMM,SpMM,GEMM>) the row of nonzero (i,j) is
+// X(j,:) = F(j,:) scaled by y = vals <Cq(i,:), X2(j,:)>: the item's row of Cq
+// stays in registers, the dot product is summed across the group by shuffles.
+template <int K, int VPL, int GS, int R, bool PF, bool H, bool S, typename Place>
 __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, int rp0, int rp1, int2 rdst,
                                            const int32_t* __restrict__ crd, const float* __restrict__ vals,
-                                           const float* __restrict__ X, const float* __restrict__ X2, int col,
-                                           Place& pl) {
-  constexpr int B0 = (H ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (H ? kBatch / 2 : kBatch) * 4 / VPL : 1;  // the same registers for any row width and with H
+                                           const float* __restrict__ X, const float* __restrict__ X2,
+                                           const float* __restrict__ Cq, int col, Place& pl) {
+  constexpr bool TWO = H || S;  // two gathered rows per nonzero
+  constexpr int B0 = (TWO ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (TWO ? kBatch / 2 : kBatch) * 4 / VPL : 1;  // the same registers for any row width and with two rows
   constexpr int B = B0 < GS ? B0 : GS;
   static_assert(GS % B == 0, "batches tile a chunk");
   constexpr int LPR = K * 4 / 128 > 0 ? K * 4 / 128 : 1;  // 128-byte lines per gathered row
@@ -442,8 +484,9 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
   };
   auto load_idx = [&](int r, int q, int& ic, float& iv) {
     const bool ok = r < R && q + gl < p1_of(r);
-    ic = ok ? __ldg(crd + q + gl) : -1;
-    iv = ok ? __ldg(vals + q + gl) : 0.f;
+    const uint64_t pol = stream_policy();
+    ic = ok ? ld_stream(crd + q + gl, pol) : -1;
+    iv = ok ? ld_stream(vals + q + gl, pol) : 0.f;
   };
   int r = 0, q = p0_of(0);  // current chunk
   int rn = r, qn = q;       // next chunk
@@ -456,6 +499,14 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
   load_idx(rn, qn, nc, nv);
   float acc[VPL];
   zero_vec(acc);
+  float crow[S ? VPL : 1];  // S: Cq's row of the current item
+  auto load_crow = [&](int rr) {
+    if constexpr (S) {
+      const int row = __shfl_sync(gmask, rdst.x, gbase + (rr < R ? rr : 0));
+      if (rr < R && row >= 0) ldg_vec<VPL>(crow, Cq + (int64_t)row * K + col); else zero_vec(crow);
+    }
+  };
+  load_crow(0);
 #pragma unroll 1
   while (r < R) {
     if constexpr (PF) {
@@ -463,7 +514,7 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
 #pragma unroll
         for (int l = 0; l < LPR; ++l) {
           prefetch_line(X + (int64_t)nc * K + 32 * l);
-          if constexpr (H) prefetch_line(X2 + (int64_t)nc * K + 32 * l);
+          if constexpr (TWO) prefetch_line(X2 + (int64_t)nc * K + 32 * l);
         }
       load_idx(r2, q2, n2c, n2v);  // two chunks ahead
     }
@@ -471,16 +522,42 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
 #pragma unroll 1
     for (int u0 = 0; u0 < m; u0 += B) {
       float x[B][VPL];
+      if constexpr (S) {
+        float d[B][VPL];
 #pragma unroll
-      for (int k = 0; k < B; ++k) {
-        const int c = __shfl_sync(gmask, ic, gbase + u0 + k);
-        if (c >= 0) gathered_row<K, VPL, H>(x[k], X, X2, c, col); else zero_vec(x[k]);
-      }
+        for (int k = 0; k < B; ++k) {
+          const int c = __shfl_sync(gmask, ic, gbase + u0 + k);
+          if (c >= 0) {
+            ldg_vec<VPL>(x[k], X + (int64_t)c * K + col);
+            ldg_vec<VPL>(d[k], X2 + (int64_t)c * K + col);
+          } else {
+            zero_vec(x[k]);
+            zero_vec(d[k]);
+          }
+        }
 #pragma unroll
-      for (int k = 0; k < B; ++k) {
-        const float v = __shfl_sync(gmask, iv, gbase + u0 + k);
+        for (int k = 0; k < B; ++k) {
+          float dot = 0.f;
 #pragma unroll
-        for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v, x[k][e], acc[e]);
+          for (int e = 0; e < VPL; ++e) dot = fmaf(crow[e], d[k][e], dot);
+#pragma unroll
+          for (int o = GS / 2; o > 0; o >>= 1) dot += __shfl_xor_sync(gmask, dot, o);
+          const float y = __shfl_sync(gmask, iv, gbase + u0 + k) * dot;
+#pragma unroll
+          for (int e = 0; e < VPL; ++e) acc[e] = fmaf(y, x[k][e], acc[e]);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < B; ++k) {
+          const int c = __shfl_sync(gmask, ic, gbase + u0 + k);
+          if (c >= 0) gathered_row<K, VPL, H>(x[k], X, X2, c, col); else zero_vec(x[k]);
+        }
+#pragma unroll
+        for (int k = 0; k < B; ++k) {
+          const float v = __shfl_sync(gmask, iv, gbase + u0 + k);
+#pragma unroll
+          for (int e = 0; e < VPL; ++e) acc[e] = fmaf(v, x[k][e], acc[e]);
+        }
       }
     }
     if (rn != r) {  // the item's last chunk: its T row is complete
@@ -490,6 +567,7 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
       if (gl == r) pl.put_dest(sl, rdst);
       pl.publish(sl, 1);
       zero_vec(acc);
+      if constexpr (S) load_crow(rn);
     }
     r = rn;
     q = qn;
@@ -649,8 +727,8 @@ template <int K, int L, int MODE, bool PF>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_gemm(WsHeader* hdr, const int4* __restrict__ segs, int max_segs,
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
-              const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ D,
-              float* __restrict__ A, float* __restrict__ partial, long long wait_cycles) {
+              const float* __restrict__ X, const float* __restrict__ X2, const float* __restrict__ Cq,
+              const float* __restrict__ D, float* __restrict__ A, float* __restrict__ partial, long long wait_cycles) {
   static_assert(K == 16 || K == 32 || K == 64 || K == 128 || K == 256, "K must be 16, 32, 64, 128 or 256");
   static_assert(L % 16 == 0 && L >= 16 && L <= 256, "L must be a multiple of 16 in [16, 256]");
   constexpr int KT = tc_kt(K);  // tile columns (K, or 32 with zero padding)
@@ -810,7 +888,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         constexpr int W2 = R < BW / 2 ? R : (BW / 2 > 1 ? BW / 2 : 1);
         constexpr int W4 = R < BW / 4 ? R : (BW / 4 > 1 ? BW / 4 : 1);
         const int n0 = __shfl_sync(gmask, rp1 - rp0, gbase);
-        if (n0 <= 1) {
+        if (MODE == kSampled) {  // items one after the other (each keeps its C row)
+          ok = long_items<K, VPL, GS, R, PF, false, true>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, Cq,
+                                                           col, pl);
+        } else if (n0 <= 1) {
 #pragma unroll 1
           for (int w0 = 0; w0 < R && ok; w0 += W1)
             ok = short_wave<K, VPL, GS, W1, 1, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
@@ -823,7 +904,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int w0 = 0; w0 < R && ok; w0 += W4)
             ok = short_wave<K, VPL, GS, W4, 4, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
         } else {
-          ok = long_items<K, VPL, GS, R, PF, H>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, col, pl);
+          ok = long_items<K, VPL, GS, R, PF, H, false>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, nullptr,
+                                                        col, pl);
         }
       }
       if (!__all_sync(0xffffffffu, ok)) break;
@@ -902,7 +984,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const int r = RPI * i + lane / LPRW, part = lane % LPRW;
           const float4 x = *reinterpret_cast<const float4*>(st + (size_t)r * PITCH + 16 * part);
           float* d = g_tc.epi_dst[q][r];
-          if (d != nullptr) *reinterpret_cast<float4*>(d + c + 4 * part) = x;
+          if (d != nullptr) st_stream(d + c + 4 * part, x, stream_policy());
         }
         stage_i = (stage_i + 1) % NSTAGE;  // with one stage, the next chunk's
         if (NSTAGE == 1) __syncwarp();     // stores wait for these reads
@@ -975,7 +1057,7 @@ cudaError_t tc_setup(TcLaunch* out) {
 template <int MODE, bool PF>
 cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const int4* segs,
                         int max_segs, int64_t dense_rows, const int32_t* crd, const float* vals, const float* X,
-                        const float* X2, const float* D, float* A, float* partial, cudaStream_t s) {
+                        const float* X2, const float* Cq, const float* D, float* A, float* partial, cudaStream_t s) {
   const long long wait = wait_limit_cycles();
 #define SLNR_TC_CASE(KK, LL)                                                                              \
   if (K == KK && L == LL) {                                                                               \
@@ -988,8 +1070,14 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
     if ((e = cudaMemsetAsync(&hdr->next_tile, 0, sizeof(int), s)) != cudaSuccess) return e;               \
     k_tc_gemm<KK, LL, MODE, PF><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,          \
                                                                              dense_rows, crd, vals, X,    \
-                                                                             X2, D, A, partial, wait);    \
+                                                                             X2, Cq, D, A, partial, wait);\
     return cudaGetLastError();                                                                            \
+  }
+  if constexpr (MODE == kSampled) {  // <SDDMM,SpMM,GEMM>: the widths of the benchmark range
+    SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128)
+    SLNR_TC_CASE(64, 32) SLNR_TC_CASE(64, 64) SLNR_TC_CASE(64, 128)
+    SLNR_TC_CASE(128, 32) SLNR_TC_CASE(128, 64) SLNR_TC_CASE(128, 128)
+    return cudaErrorInvalidValue;
   }
   SLNR_TC_CASE(16, 16) SLNR_TC_CASE(16, 32) SLNR_TC_CASE(16, 64) SLNR_TC_CASE(16, 128) SLNR_TC_CASE(16, 256)
   SLNR_TC_CASE(32, 16) SLNR_TC_CASE(32, 32) SLNR_TC_CASE(32, 64) SLNR_TC_CASE(32, 128) SLNR_TC_CASE(32, 256)
@@ -1045,19 +1133,32 @@ cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, 
   const bool pf = (size_t)B.ncols * (size_t)K * sizeof(float) * (C2 != nullptr ? 2 : 1) > l2_bytes() / 2;
   if (C2 != nullptr)
     return pf ? tc_dispatch<kSegmentsH, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                              B.vals, C, C2, D, A, plan.partial, s)
+                                              B.vals, C, C2, nullptr, D, A, plan.partial, s)
               : tc_dispatch<kSegmentsH, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                               B.vals, C, C2, D, A, plan.partial, s);
+                                               B.vals, C, C2, nullptr, D, A, plan.partial, s);
   return pf ? tc_dispatch<kSegments, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                           B.vals, C, nullptr, D, A, plan.partial, s)
+                                           B.vals, C, nullptr, nullptr, D, A, plan.partial, s)
             : tc_dispatch<kSegments, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                            B.vals, C, nullptr, D, A, plan.partial, s);
+                                            B.vals, C, nullptr, nullptr, D, A, plan.partial, s);
+}
+
+bool tc_sampled_supported(int K, int L, int M) {
+  return K == L && (L == 32 || L == 64 || L == 128) && (M == 32 || M == 64 || M == 128);
+}
+
+cudaError_t launch_tc_sddmm_spmm_gemm(const CsrView& B, const float* C, const float* D, const float* F, int L,
+                                      const float* W, int M, float* A, const SegPlan& plan, cudaStream_t s) {
+  if (B.nrows <= 0) return cudaSuccess;
+  // T rows of width L: the gathered row is F(j,:), its scale C(i,:).D(j,:)
+  return tc_dispatch<kSampled, false>(L, M, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, F,
+                                      D, C, W, A, plan.partial, s);
 }
 
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  return tc_dispatch<kDense, false>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, D, A, nullptr, s);
+  return tc_dispatch<kDense, false>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, nullptr, D, A, nullptr,
+                                    s);
 }
 
 }  // namespace slnr

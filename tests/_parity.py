@@ -61,12 +61,13 @@ def values_of(op, out):
 
 def uses_tensor_cores(op, variant="fused") -> bool:
     """Whether the call may contract on TF32 tensor cores when allowed: the
-    fused and unfused <SpMM,GEMM>, <SpTTM,SpTTM> and <SpMMH,GEMM>, and the
-    dense GEMM of the unfused <SDDMM,SpMM,GEMM> and <MTTKRP,GEMM> (their fused
-    consumers run in fp32)."""
-    if op in ("spmm_gemm", "spttm_ttm", "spmmh_gemm"):
+    fused and unfused <SpMM,GEMM>, <SpTTM,SpTTM>, <SpMMH,GEMM> and
+    <SDDMM,SpMM,GEMM> (fused: where the dot product and the temporary have
+    one width), and the dense GEMM of the unfused <MTTKRP,GEMM> (its fused
+    consumer runs in fp32)."""
+    if op in ("spmm_gemm", "spttm_ttm", "spmmh_gemm", "sddmm_spmm_gemm"):
         return True
-    return variant == "unfused" and op in ("sddmm_spmm_gemm", "mttkrp_gemm")
+    return variant == "unfused" and op == "mttkrp_gemm"
 
 
 def tolerance(op, allow_tf32, variant="fused") -> float:

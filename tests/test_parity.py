@@ -93,7 +93,8 @@ def test_mttkrp_hub_slice(slnr, orc, L, variant):
                                  (128, 256), (256, 128)])
 @pytest.mark.parametrize("variant", ["fused", "unfused"])
 def test_spttm_ttm_widths(slnr, orc, L, M, variant):
-    w = wl.spttm_ttm_powerlaw(0x51A4 + L + M, (60, 70, 900), 12000, 8.0, 900, L, M)
+    # 24000 nonzeros: past the size below which the fused call stays on CUDA cores
+    w = wl.spttm_ttm_powerlaw(0x51A4 + L + M, (100, 100, 900), 24000, 8.0, 900, L, M)
     check(slnr, orc, w, variant, False)
     check(slnr, orc, w, variant, True)
 
@@ -254,9 +255,9 @@ def test_gathered_matrix_larger_than_l2(slnr, orc, K, L):
 
 @pytest.mark.parametrize("K,L", [(16, 16), (32, 64), (128, 128), (128, 256)])
 @pytest.mark.parametrize("nrows", [1, 3, 130])
-def test_tensor_core_path_on_tiny_inputs(slnr, orc, K, L, nrows):
-    # fewer rows than one 128-row tile, exactly one tile plus a ragged second:
-    # the dynamic tile counter hands out one or two tiles to a full grid of CTAs
+def test_tiny_inputs(slnr, orc, K, L, nrows):
+    # fewer rows than one 128-row tile, exactly one tile plus a ragged second
+    # (below 2^14 nonzeros the fused call runs on the CUDA-core kernels)
     w = wl.spmm_gemm_uniform(0x51A4 + 13 * K + L + nrows, nrows, 300, 7, K, L, name=f"tiny_{nrows}")
     check(slnr, orc, w, "fused", True)
     check(slnr, orc, w, "unfused", True)
@@ -274,3 +275,24 @@ def test_single_buffer_tensor_core_path(slnr, orc, K, L, op):
     else:
         w = wl.spttm_ttm_powerlaw(0x51A4 + 23 * K + L, (200, 200, 900), 100000, 8.0, 900, K, L)
     check(slnr, orc, w, "fused", True)
+
+
+@pytest.mark.parametrize("op,size", [("spmm_gemm", "small"), ("spmm_gemm", "large"),
+                                     ("sddmm_spmm_gemm", "small"), ("sddmm_spmm_gemm", "large")])
+def test_fused_call_routing(slnr, orc, op, size):
+    # the fused call takes the tensor-core kernel from 2^14 nonzeros on (TF32
+    # allowed, supported widths) and the CUDA-core kernels below; both agree
+    # with the oracle
+    n, deg = (1024, 10) if size == "small" else (4000, 12)
+    w = wl.spmm_gemm_rmat(0x51A4 + 97, n, deg, 64, 64) if op == "spmm_gemm" else \
+        wl.sddmm_spmm_gemm_rmat(0x51A4 + 98, n, deg, 64, 64, 64)
+    nnz = len(w.B.crd)
+    assert (nnz < (1 << 14)) == (size == "small")
+    slnr.timing_enable(True)
+    try:
+        check(slnr, orc, w, "fused", True)
+        names = [name for name, _ in slnr.timing_read()]
+    finally:
+        slnr.timing_enable(False)
+    on_tc = any(name.startswith("tc_") for name in names)
+    assert on_tc == (size == "large"), names
