@@ -303,6 +303,10 @@ __host__ __device__ constexpr size_t tc_smem_bytes(int K, int L) {
 #define SLNR_TC_BATCH 4  // gathered rows a lane group keeps in flight (one batch; half with Hadamard rows)
 #endif
 constexpr int kBatch = SLNR_TC_BATCH;
+#ifndef SLNR_TC_SHORT_BATCH
+#define SLNR_TC_SHORT_BATCH 8  // rows in flight in a wave of short items (they need no accumulator of their own)
+#endif
+constexpr int kShortBatch = SLNR_TC_SHORT_BATCH;
 
 #ifndef SLNR_TC_STREAM_HINT
 #define SLNR_TC_STREAM_HINT 1  // 1: streamed loads and stores carry an L2 evict-first hint
@@ -353,7 +357,7 @@ struct ProdLayout {
   static constexpr int VPL = K > 128 ? 8 : 4;  // a group is at most a warp
   static constexpr int GS = K / VPL;
   static constexpr int G = 32 / GS;
-  static constexpr int R = GS < kBatch ? GS : kBatch;
+  static constexpr int R = GS < kShortBatch ? GS : kShortBatch;
   static constexpr int IPC = G * R;
   static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
   static_assert(kTcRows % IPC == 0, "claims tile the item tile");
@@ -414,7 +418,7 @@ __device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, in
                                            Place& pl) {
   constexpr int S = W * N;                // row slots of the batch
   constexpr int SPL = (S + GS - 1) / GS;  // slots loaded per lane
-  static_assert(S <= kBatch, "a wave is one batch");
+  static_assert(S <= kShortBatch, "a wave is one batch");
   int mc[SPL];
   float mv[SPL];
 #pragma unroll
@@ -883,7 +887,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // item0 has more nonzeros than item0's class bound, so item0 picks
         // the wave shape for the group's R items.
         // rows in flight per group: fewer with two loads each (H) or 8 columns per lane
-        constexpr int BW = (H ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (H ? kBatch / 2 : kBatch) * 4 / VPL : 1;
+        constexpr int BW = (H ? kShortBatch / 2 : kShortBatch) * 4 / VPL > 0
+                               ? (H ? kShortBatch / 2 : kShortBatch) * 4 / VPL : 1;
         constexpr int W1 = R < BW ? R : BW;
         constexpr int W2 = R < BW / 2 ? R : (BW / 2 > 1 ? BW / 2 : 1);
         constexpr int W4 = R < BW / 4 ? R : (BW / 4 > 1 ? BW / 4 : 1);
