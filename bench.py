@@ -177,11 +177,40 @@ def consumer_flops(w) -> int:
     return 0
 
 
+def gather_bytes(w) -> int:
+    """Bytes the fused producers read as whole gathered rows, one (or two)
+    per nonzero and one per fiber where a fiber scales a row: nnz 4K for
+    <SpMM,GEMM>, nnz 4L for <SpTTM,SpTTM>, nnz 8J for <SpMMH,GEMM>, nnz 4(L+K)
+    for <SDDMM,SpMM>, nnz 4(K+L) for <SDDMM,SpMM,GEMM>, (nnz + nfibers) 4L for
+    MTTKRP.  Almost all of them hit in L2; their rate, not HBM's, is the
+    realistic ceiling of the gathering kernels."""
+    d, B = w.dims, w.B
+    per_nnz = {"spmm_gemm": lambda: 4 * d["K"], "spttm_ttm": lambda: 4 * d["L"], "spmmh_gemm": lambda: 8 * d["J"],
+               "sddmm_spmm": lambda: 4 * (d["L"] + d["K"]), "sddmm_spmm_gemm": lambda: 4 * (d["K"] + d["L"]),
+               "mttkrp": lambda: 4 * d["L"], "mttkrp_gemm": lambda: 4 * d["L"]}[w.op]()
+    extra = 4 * d["L"] * B.nfibers if w.op in ("mttkrp", "mttkrp_gemm") else 0
+    return int(per_nnz * B.nnz + extra)
+
+
+def gather_row_width(w) -> int:
+    """Width (fp32 values) of the rows the producers gather, as a power of two
+    in [4, 128] for the gather peak kernel."""
+    d = w.dims
+    width = {"spmm_gemm": "K", "spttm_ttm": "L", "spmmh_gemm": "J", "sddmm_spmm": "K", "sddmm_spmm_gemm": "L",
+             "mttkrp": "L", "mttkrp_gemm": "L"}[w.op]
+    v = 4
+    while v * 2 <= min(d[width], 128):
+        v *= 2
+    return v
+
+
 def kernel_source_hash() -> str:
+    """Hash of the kernel sources that run inside the measured calls (the
+    peak-measuring kernels of peaks.cu run outside them)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2205_11622_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
+        if name.endswith((".cu", ".cuh", ".h")) and name != "peaks.cu":
             h.update(name.encode())
             h.update(open(os.path.join(csrc, name), "rb").read())
     return h.hexdigest()[:16]
@@ -511,7 +540,8 @@ def main():
     achieved = mbytes[dom] / (k_ms / 1e3) / 1e9
     all_rows = min_bytes_all_rows(dw)
     traffic = ncu_traffic(dw.name)
-    pk = slnr.peaks(stream) if rank == 0 else {}
+    pk = slnr.peaks(stream, gather_width=gather_row_width(dw)) if rank == 0 else {}
+    gb = gather_bytes(dw)
     cflops = consumer_flops(dw)
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "traffic": traffic,
@@ -527,7 +557,15 @@ def main():
                             "tf32_frac": round(cflops / (k_ms / 1e3) / 1e12 / pk["tf32_tflops"], 4)
                             if pk.get("tf32_tflops") else None,
                             "note": "the dense consumer contraction of the dominant kernel (2 K L per non-empty "
-                                    "row) against this library's own tcgen05 kind::tf32 peak kernel"}}
+                                    "row) against this library's own tcgen05 kind::tf32 peak kernel"},
+                "gather": {"bytes": gb, "unit": "GB/s", "achieved": round(gb / (k_ms / 1e3) / 1e9, 1),
+                           "l2_gather_peak_measured": round(pk.get("l2_gather_gbs", 0.0), 1),
+                           "hbm_gather_peak_measured": round(pk.get("hbm_gather_gbs", 0.0), 1),
+                           "frac_l2": round(gb / (k_ms / 1e3) / 1e9 / pk["l2_gather_gbs"], 4)
+                           if pk.get("l2_gather_gbs") else None,
+                           "row_width": gather_row_width(dw),
+                           "note": "whole rows the producers gather (one per nonzero), against this library's own "
+                                   "row-gather kernel on an L2-resident table (a quarter of L2) and on a 2 GB table"}}
 
     cpu = None
     if rank == 0 and world == 1 and not args.skip_cpu:

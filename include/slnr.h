@@ -266,6 +266,19 @@ slnr_status slnr_set_wait_limit(int64_t cycles);
 slnr_status slnr_peak_ffma(void *stream, double *tflops);
 slnr_status slnr_peak_tf32(void *stream, double *tflops);
 
+/* The rate of whole-row gathers, the loads the fused producers issue for
+ * each nonzero (Sec. 6.3: the fused <SpMM,GEMM> reads one row of C per
+ * nonzero), in GB/s: lane groups of width/4 lanes read rows of the caller's
+ * device table (rows x width fp32, row-major, 16-byte aligned, contents
+ * arbitrary; not written) at pseudo-random row ids, 8 rows in flight per
+ * group, about 4 GB per launch; a second, timed launch follows a first one.
+ * A table that fits in L2 gives the L2 gather rate, a larger one the HBM
+ * gather rate.  width is a power of two in [4, 128] and rows in
+ * [1, 2^31) (SLNR_ERR_SHAPE otherwise); a misaligned table returns
+ * SLNR_ERR_UNSUPPORTED.  Runs on `stream` and waits for it; allocates
+ * nothing. */
+slnr_status slnr_peak_gather(const float *table, int64_t rows, int width, void *stream, double *gbs);
+
 /* ---- diagnostics ------------------------------------------------------- */
 const char *slnr_status_string(slnr_status status);
 /* Detail of the last error raised on the calling thread ("" if none). */

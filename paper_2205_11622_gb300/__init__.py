@@ -74,6 +74,7 @@ SIGNATURES = {
     "slnr_set_wait_limit": ([ctypes.c_int64], ctypes.c_int),
     "slnr_peak_ffma": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "slnr_peak_tf32": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+    "slnr_peak_gather": ([_P, ctypes.c_int64, ctypes.c_int, _P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
     "slnr_timing_get": ([_I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
@@ -121,15 +122,32 @@ def timing_enable(on: bool = True):
     _check(lib().slnr_timing_enable(int(bool(on))), "slnr_timing_enable")
 
 
-def peaks(stream=None):
-    """{"ffma_tflops", "tf32_tflops"}: the compute peaks measured by the library's own kernels."""
+def peaks(stream=None, gather_width=None):
+    """{"ffma_tflops", "tf32_tflops"}: the compute peaks measured by the library's own kernels.
+
+    With gather_width (a power of two in [4, 128]) also "l2_gather_gbs" and
+    "hbm_gather_gbs": the rate of whole-row gathers of that width from a
+    table of a quarter of L2 and from one of 2 GB (slnr_peak_gather)."""
     torch = _torch()
-    s = ctypes.c_void_p((stream or torch.cuda.current_stream()).cuda_stream)
+    st = stream or torch.cuda.current_stream()
+    s = ctypes.c_void_p(st.cuda_stream)
     out = {}
     for key, fn in (("ffma_tflops", "slnr_peak_ffma"), ("tf32_tflops", "slnr_peak_tf32")):
         v = ctypes.c_double(0.0)
         _check(getattr(lib(), fn)(s, ctypes.byref(v)), fn)
         out[key] = v.value
+    if gather_width is not None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+        l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+        for key, nbytes in (("l2_gather_gbs", l2 // 4), ("hbm_gather_gbs", 2 << 30)):
+            rows = nbytes // (4 * gather_width)
+            with torch.cuda.stream(st):
+                table = torch.zeros((rows, gather_width), dtype=torch.float32, device=dev)
+            v = ctypes.c_double(0.0)
+            _check(lib().slnr_peak_gather(ctypes.c_void_p(table.data_ptr()), rows, gather_width, s,
+                                          ctypes.byref(v)), "slnr_peak_gather")
+            out[key] = v.value
+            del table
     return out
 
 

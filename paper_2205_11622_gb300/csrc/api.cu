@@ -435,6 +435,16 @@ slnr_status slnr_peak_tf32(void* stream, double* tflops) {
   return SLNR_OK;
 }
 
+slnr_status slnr_peak_gather(const float* table, int64_t rows, int width, void* stream, double* gbs) {
+  if (!table || !gbs) return fail(SLNR_ERR_NULL, "table or gbs is NULL");
+  if (rows < 1 || rows > INT32_MAX) return fail(SLNR_ERR_SHAPE, "rows must be in [1, 2^31)");
+  if (width < 4 || width > 128 || (width & (width - 1)) != 0)
+    return fail(SLNR_ERR_SHAPE, "width must be a power of two in [4, 128]");
+  if (!aligned16(table)) return fail(SLNR_ERR_UNSUPPORTED, "table must be 16-byte aligned");
+  SLNR_CUDA(peak_gather(table, rows, width, static_cast<cudaStream_t>(stream), gbs));
+  return SLNR_OK;
+}
+
 slnr_status slnr_set_wait_limit(int64_t cycles) {
   if (cycles < 0) return fail(SLNR_ERR_SHAPE, "wait limit must be >= 0");
   g_wait_limit = cycles;

@@ -157,9 +157,11 @@ cudaError_t launch_w_mttkrp_units(int L, const slnr_csf3& B, const float* C, con
 cudaError_t launch_w_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& plan, const float* E, int M, float* A,
                                     cudaStream_t s);
 
-// peaks.cu -- compute peaks measured by the library's own kernels (TFLOP/s)
+// peaks.cu -- peaks measured by the library's own kernels (TFLOP/s, GB/s)
 cudaError_t peak_ffma(cudaStream_t s, double* tflops);
 cudaError_t peak_tf32(cudaStream_t s, double* tflops);
+// rows x width fp32 table (width in {4, 8, ..., 128}, 16-byte aligned); GB/s of row gathers
+cudaError_t peak_gather(const float* table, int64_t rows, int width, cudaStream_t s, double* gbs);
 
 }  // namespace slnr
 

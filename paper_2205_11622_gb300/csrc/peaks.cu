@@ -1,7 +1,10 @@
-// Compute peaks of this GPU, measured by the library's own kernels: the
-// FP32 FFMA rate of the CUDA cores and the TF32 rate of the tcgen05 tensor
-// cores (the two kinds of arithmetic the consumer contractions run on).
-// They are the compute denominators of the roofline the benchmark reports.
+// Peaks of this GPU, measured by the library's own kernels: the FP32 FFMA
+// rate of the CUDA cores and the TF32 rate of the tcgen05 tensor cores (the
+// two kinds of arithmetic the consumer contractions run on), and the rate of
+// whole-row gathers from a table (the producers' loads).  They are the
+// compute and gather denominators of the roofline the benchmark reports.
+#include <algorithm>
+
 #include "launch.h"
 #include "tcgen05.cuh"
 
@@ -87,6 +90,41 @@ __global__ void __launch_bounds__(128, 1) k_peak_tf32(int64_t passes) {
   if (warp == 0) tc::tmem_dealloc(tmem, kMmaN);
 }
 
+constexpr int kGatherThreads = 256;
+constexpr int kGatherBatch = 8;  // rows in flight per lane group
+
+// Row gathers, as the producers of the fused kernels issue them: a lane group
+// of q = width / 4 lanes reads a whole row of a rows x width fp32 table (one
+// float4 per lane) at a pseudo-random row id, kGatherBatch rows in flight,
+// and keeps a running sum.  Row ids come from a per-group linear
+// congruential sequence (the Numerical Recipes constants) mapped to
+// [0, rows) by a multiply-shift.  `sink` is written only if the sum equals
+// a given number, so the loads cannot be dropped.
+__global__ void __launch_bounds__(kGatherThreads) k_peak_gather(const float4* __restrict__ table, uint32_t rows,
+                                                                int q, int iters, float* sink) {
+  const int lane = threadIdx.x & 31, g = lane / q, c = lane % q;
+  const uint32_t group = (blockIdx.x * (kGatherThreads / 32) + (threadIdx.x >> 5)) * (32 / q) + g;
+  uint32_t x = group * 0x9E3779B9u + 0x7F4A7C15u;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = 0; i < iters; ++i) {
+    float4 v[kGatherBatch];
+#pragma unroll
+    for (int u = 0; u < kGatherBatch; ++u) {
+      x = x * 1664525u + 1013904223u;
+      const uint32_t r = (uint32_t)(((uint64_t)(x ^ (x >> 16)) * rows) >> 32);
+      v[u] = __ldg(table + (int64_t)r * q + c);
+    }
+#pragma unroll
+    for (int u = 0; u < kGatherBatch; ++u) {
+      acc.x += v[u].x;
+      acc.y += v[u].y;
+      acc.z += v[u].z;
+      acc.w += v[u].w;
+    }
+  }
+  if (sink != nullptr && acc.x + acc.y + acc.z + acc.w == 1234.5f) sink[0] = acc.x;
+}
+
 template <typename F>
 cudaError_t timed(cudaStream_t s, float* ms, F launch) {
   cudaEvent_t a, b;
@@ -140,6 +178,24 @@ cudaError_t peak_tf32(cudaStream_t s, double* tflops) {
   if ((e = cudaMemcpyFromSymbol(&flag, g_peak_flag, sizeof(int))) != cudaSuccess) return e;
   if (flag != 0) return cudaErrorLaunchTimeout;
   *tflops = 2.0 * kMmaM * kMmaN * 8 * 4 * (double)passes * grid / (ms * 1e-3) / 1e12;
+  return cudaSuccess;
+}
+
+cudaError_t peak_gather(const float* table, int64_t rows, int width, cudaStream_t s, double* gbs) {
+  const int q = width / 4;
+  const int grid = device_sm_count() * (2048 / kGatherThreads);
+  const int64_t groups = (int64_t)grid * (kGatherThreads / 32) * (32 / q);
+  const int64_t row_bytes = (int64_t)width * 4;
+  // about 4 GB of gathered rows per launch
+  const int iters = (int)std::max<int64_t>(1, ((int64_t)4 << 30) / (groups * kGatherBatch * row_bytes));
+  float ms = 0.f;
+  cudaError_t e = timed(s, &ms, [&] {
+    k_peak_gather<<<grid, kGatherThreads, 0, s>>>(reinterpret_cast<const float4*>(table), (uint32_t)rows, q, iters,
+                                                  nullptr);
+    return cudaGetLastError();
+  });
+  if (e != cudaSuccess) return e;
+  *gbs = (double)groups * iters * kGatherBatch * row_bytes / (ms * 1e-3) / 1e9;
   return cudaSuccess;
 }
 

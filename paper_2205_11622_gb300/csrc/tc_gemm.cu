@@ -349,15 +349,18 @@ __device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("pre
 // Producer lane layout: a T row is built by a group of GS = K / 4 lanes (at
 // most a warp), lane gl of the group holding the 4 columns [4 gl, 4 gl + 4)
 // as one float4; a warp holds G = 32 / GS groups.  A claim is IPC = G * R
-// consecutive items of an item tile, group g taking items g R .. g R + R - 1
-// (R more items per group where the rows are narrow, so a claim is at
-// least 8 items).
-template <int K>
+// consecutive items of an item tile, group g taking items g R .. g R + R - 1,
+// with R = min(GS, RB) (a lane of the group holds each item's record).  RB is
+// the short-wave width, or the long-item batch where every item runs on its
+// own (sampled rows: claims of 8 such items made the tiles of heavy-row
+// chunks at the head of the list twice as long).
+template <int K, bool SEQ>
 struct ProdLayout {
   static constexpr int VPL = K > 128 ? 8 : 4;  // a group is at most a warp
   static constexpr int GS = K / VPL;
   static constexpr int G = 32 / GS;
-  static constexpr int R = GS < kShortBatch ? GS : kShortBatch;
+  static constexpr int RB = SEQ ? kBatch : kShortBatch;
+  static constexpr int R = GS < RB ? GS : RB;
   static constexpr int IPC = G * R;
   static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
   static_assert(kTcRows % IPC == 0, "claims tile the item tile");
@@ -736,7 +739,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   static_assert(K == 16 || K == 32 || K == 64 || K == 128 || K == 256, "K must be 16, 32, 64, 128 or 256");
   static_assert(L % 16 == 0 && L >= 16 && L <= 256, "L must be a multiple of 16 in [16, 256]");
   constexpr int KT = tc_kt(K);  // tile columns (K, or 32 with zero padding)
-  using PL = ProdLayout<K>;
+  using PL = ProdLayout<K, MODE == kSampled>;
   constexpr int NBUF = tc_nbuf(K, L);
   constexpr uint32_t IDESC = tc::idesc_tf32(kTcRows, L);
   // TMEM columns: NBUF fp32 accumulators of L columns; an allocation is a
