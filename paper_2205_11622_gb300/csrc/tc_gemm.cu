@@ -343,8 +343,6 @@ __device__ __forceinline__ void st_stream(float* p, float4 x, uint64_t pol) {
                : "memory");
 }
 
-// L2 prefetch of the 128-byte line holding p (no register, nothing to wait for).
-__device__ __forceinline__ void prefetch_line(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 
 // Producer lane layout: a T row is built by a group of GS = K / 4 lanes (at
 // most a warp), lane gl of the group holding the 4 columns [4 gl, 4 gl + 4)
@@ -462,13 +460,13 @@ __device__ __forceinline__ bool short_wave(unsigned gmask, int gbase, int gl, in
 // nonzeros are walked in chunks of GS (a chunk never spans two items): lane
 // t holds the coordinate and value of nonzero t of the current chunk, and the
 // next chunk's (which may be the next item's first) are loaded while this one
-// is gathered.  With PF the chunk after that is loaded too, and the rows of
-// the next chunk are prefetched into L2 (one lane per row,
-// prefetch.global.L2, no register held) while this chunk is gathered.
+// is gathered.  (Prefetching the next chunk's rows into L2 as well raised the
+// DRAM traffic of gathered matrices larger than L2: lines arrived early and
+// were evicted before use.)
 // With S (sampled rows, <SDDMM,SpMM,GEMM>) the row of nonzero (i,j) is
 // X(j,:) = F(j,:) scaled by y = vals <Cq(i,:), X2(j,:)>: the item's row of Cq
 // stays in registers, the dot product is summed across the group by shuffles.
-template <int K, int VPL, int GS, int R, bool PF, bool H, bool S, typename Place>
+template <int K, int VPL, int GS, int R, bool H, bool S, typename Place>
 __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, int rp0, int rp1, int2 rdst,
                                            const int32_t* __restrict__ crd, const float* __restrict__ vals,
                                            const float* __restrict__ X, const float* __restrict__ X2,
@@ -477,7 +475,6 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
   constexpr int B0 = (TWO ? kBatch / 2 : kBatch) * 4 / VPL > 0 ? (TWO ? kBatch / 2 : kBatch) * 4 / VPL : 1;  // the same registers for any row width and with two rows
   constexpr int B = B0 < GS ? B0 : GS;
   static_assert(GS % B == 0, "batches tile a chunk");
-  constexpr int LPR = K * 4 / 128 > 0 ? K * 4 / 128 : 1;  // 128-byte lines per gathered row
   auto p0_of = [&](int r) { return __shfl_sync(gmask, rp0, gbase + r); };
   auto p1_of = [&](int r) { return __shfl_sync(gmask, rp1, gbase + r); };
   // a chunk is item r's nonzeros [q, min(q + GS, p1(r))); r == R: none left
@@ -498,10 +495,8 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
   int r = 0, q = p0_of(0);  // current chunk
   int rn = r, qn = q;       // next chunk
   advance(rn, qn);
-  int r2 = rn, q2 = qn;     // the chunk after (PF)
-  if (PF) advance(r2, q2);
-  int ic, nc, n2c = -1;
-  float iv, nv, n2v = 0.f;
+  int ic, nc;
+  float iv, nv;
   load_idx(r, q, ic, iv);
   load_idx(rn, qn, nc, nv);
   float acc[VPL];
@@ -516,15 +511,6 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
   load_crow(0);
 #pragma unroll 1
   while (r < R) {
-    if constexpr (PF) {
-      if (nc >= 0)  // rows of the next chunk (coordinates loaded one chunk ago) into L2
-#pragma unroll
-        for (int l = 0; l < LPR; ++l) {
-          prefetch_line(X + (int64_t)nc * K + 32 * l);
-          if constexpr (TWO) prefetch_line(X2 + (int64_t)nc * K + 32 * l);
-        }
-      load_idx(r2, q2, n2c, n2v);  // two chunks ahead
-    }
     const int m = min(GS, p1_of(r) - q);
 #pragma unroll 1
     for (int u0 = 0; u0 < m; u0 += B) {
@@ -580,16 +566,8 @@ __device__ __forceinline__ bool long_items(unsigned gmask, int gbase, int gl, in
     q = qn;
     ic = nc;
     iv = nv;
-    if constexpr (PF) {
-      rn = r2;
-      qn = q2;
-      nc = n2c;
-      nv = n2v;
-      advance(r2, q2);
-    } else {
-      advance(rn, qn);
-      load_idx(rn, qn, nc, nv);
-    }
+    advance(rn, qn);
+    load_idx(rn, qn, nc, nv);
   }
   return true;
 }
@@ -730,7 +708,7 @@ struct Placer {
 constexpr int kProducerWarps = kTcWarps - 5;
 constexpr int kMmaWarp = kTcWarps - 5;  // then the four epilogue warps
 
-template <int K, int L, int MODE, bool PF>
+template <int K, int L, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_gemm(WsHeader* hdr, const int4* __restrict__ segs, int max_segs,
               int64_t dense_rows, const int32_t* __restrict__ crd, const float* __restrict__ vals,
@@ -897,7 +875,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         constexpr int W4 = R < BW / 4 ? R : (BW / 4 > 1 ? BW / 4 : 1);
         const int n0 = __shfl_sync(gmask, rp1 - rp0, gbase);
         if (MODE == kSampled) {  // items one after the other (each keeps its C row)
-          ok = long_items<K, VPL, GS, R, PF, false, true>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, Cq,
+          ok = long_items<K, VPL, GS, R, false, true>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, Cq,
                                                            col, pl);
         } else if (n0 <= 1) {
 #pragma unroll 1
@@ -912,7 +890,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int w0 = 0; w0 < R && ok; w0 += W4)
             ok = short_wave<K, VPL, GS, W4, 4, H>(gmask, gbase, gl, rp0, rp1, rdst, w0, crd, vals, X, X2, col, pl);
         } else {
-          ok = long_items<K, VPL, GS, R, PF, H, false>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, nullptr,
+          ok = long_items<K, VPL, GS, R, H, false>(gmask, gbase, gl, rp0, rp1, rdst, crd, vals, X, X2, nullptr,
                                                         col, pl);
         }
       }
@@ -1025,7 +1003,7 @@ struct TcLaunch {
   size_t smem;
 };
 
-template <int K, int L, int MODE, bool PF>
+template <int K, int L, int MODE>
 cudaError_t tc_setup(TcLaunch* out) {
   static TcLaunch cached[64] = {};
   int dev = 0;
@@ -1044,14 +1022,14 @@ cudaError_t tc_setup(TcLaunch* out) {
   const int max_ctas = 512 / (int)tc_tmem_cols(K, L);
   const size_t floor_bytes = (size_t)sm_smem / (size_t)(max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
-  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE, PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
+  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
       cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE, PF>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  if ((e = cudaFuncSetAttribute(k_tc_gemm<K, L, MODE>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                 (int)cudaSharedmemCarveoutMaxShared)) != cudaSuccess)
     return e;
   int occ = 0;
-  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_tc_gemm<K, L, MODE, PF>, kTcThreads, smem)) !=
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_tc_gemm<K, L, MODE>, kTcThreads, smem)) !=
       cudaSuccess)
     return e;
   if (occ < 1) return cudaErrorInvalidConfiguration;
@@ -1062,7 +1040,7 @@ cudaError_t tc_setup(TcLaunch* out) {
   return cudaSuccess;
 }
 
-template <int MODE, bool PF>
+template <int MODE>
 cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const int4* segs,
                         int max_segs, int64_t dense_rows, const int32_t* crd, const float* vals, const float* X,
                         const float* X2, const float* Cq, const float* D, float* A, float* partial, cudaStream_t s) {
@@ -1070,15 +1048,15 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
 #define SLNR_TC_CASE(KK, LL)                                                                              \
   if (K == KK && L == LL) {                                                                               \
     TcLaunch tl;                                                                                          \
-    cudaError_t e = tc_setup<KK, LL, MODE, PF>(&tl);                                                      \
+    cudaError_t e = tc_setup<KK, LL, MODE>(&tl);                                                          \
     if (e != cudaSuccess) return e;                                                                       \
     int64_t grid = (items_upper + kTcRows - 1) / kTcRows;                                                 \
     if (grid > tl.grid_cap) grid = tl.grid_cap;                                                           \
     if (grid < 1) grid = 1;                                                                               \
     if ((e = cudaMemsetAsync(&hdr->next_tile, 0, sizeof(int), s)) != cudaSuccess) return e;               \
-    k_tc_gemm<KK, LL, MODE, PF><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs,          \
-                                                                             dense_rows, crd, vals, X,    \
-                                                                             X2, Cq, D, A, partial, wait);\
+    k_tc_gemm<KK, LL, MODE><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs, dense_rows,  \
+                                                                         crd, vals, X, X2, Cq, D, A,     \
+                                                                         partial, wait);                 \
     return cudaGetLastError();                                                                            \
   }
   if constexpr (MODE == kSampled) {  // <SDDMM,SpMM,GEMM>: the widths of the benchmark range
@@ -1094,19 +1072,6 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
   SLNR_TC_CASE(256, 16) SLNR_TC_CASE(256, 32) SLNR_TC_CASE(256, 64)
 #undef SLNR_TC_CASE
   return cudaErrorInvalidValue;
-}
-
-// L2 size of the current device (cached per device; 0 if it cannot be read).
-size_t l2_bytes() {
-  static size_t cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  if (cached[dev] == 0) {
-    int v = 0;
-    if (cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev) != cudaSuccess) return 0;
-    cached[dev] = (size_t)v;
-  }
-  return cached[dev];
 }
 
 }  // namespace
@@ -1136,18 +1101,11 @@ cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t
 cudaError_t launch_tc_spmm_gemm(int K, int L, const CsrView& B, const float* C, const float* D, float* A,
                                 const SegPlan& plan, cudaStream_t s, const float* C2) {
   if (B.nrows <= 0) return cudaSuccess;
-  // Gathered rows that do not fit in half of L2 miss often: the producers
-  // then prefetch the rows of the next chunk of nonzeros into L2 (long_items).
-  const bool pf = (size_t)B.ncols * (size_t)K * sizeof(float) * (C2 != nullptr ? 2 : 1) > l2_bytes() / 2;
   if (C2 != nullptr)
-    return pf ? tc_dispatch<kSegmentsH, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                              B.vals, C, C2, nullptr, D, A, plan.partial, s)
-              : tc_dispatch<kSegmentsH, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                               B.vals, C, C2, nullptr, D, A, plan.partial, s);
-  return pf ? tc_dispatch<kSegments, true>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                           B.vals, C, nullptr, nullptr, D, A, plan.partial, s)
-            : tc_dispatch<kSegments, false>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd,
-                                            B.vals, C, nullptr, nullptr, D, A, plan.partial, s);
+    return tc_dispatch<kSegmentsH>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, C, C2,
+                                   nullptr, D, A, plan.partial, s);
+  return tc_dispatch<kSegments>(K, L, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, C,
+                                nullptr, nullptr, D, A, plan.partial, s);
 }
 
 bool tc_sampled_supported(int K, int L, int M) {
@@ -1158,15 +1116,14 @@ cudaError_t launch_tc_sddmm_spmm_gemm(const CsrView& B, const float* C, const fl
                                       const float* W, int M, float* A, const SegPlan& plan, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
   // T rows of width L: the gathered row is F(j,:), its scale C(i,:).D(j,:)
-  return tc_dispatch<kSampled, false>(L, M, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, F,
-                                      D, C, W, A, plan.partial, s);
+  return tc_dispatch<kSampled>(L, M, plan.max_segs, plan.hdr, plan.segs, plan.max_segs, 0, B.crd, B.vals, F, D, C,
+                               W, A, plan.partial, s);
 }
 
 cudaError_t launch_tc_dense_gemm(int64_t M, int K, int L, const float* T, const float* D, float* A,
                                  WsHeader* hdr, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  return tc_dispatch<kDense, false>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, nullptr, D, A, nullptr,
-                                    s);
+  return tc_dispatch<kDense>(K, L, M, hdr, nullptr, 0, M, nullptr, nullptr, T, nullptr, nullptr, D, A, nullptr, s);
 }
 
 }  // namespace slnr

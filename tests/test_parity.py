@@ -246,9 +246,9 @@ def test_explicit_stream_and_workspace(slnr, orc):
 
 @pytest.mark.parametrize("K,L", [(32, 64), (64, 64), (128, 128)])
 def test_gathered_matrix_larger_than_l2(slnr, orc, K, L):
-    # C has 2^20 rows (128-512 MB, more than half of L2): the tensor-core
-    # producers then prefetch rows ahead of their gathers; 3001 rows of 21
-    # uniform columns give partial last batches in every row
+    # C has 2^20 rows (128-512 MB, more than L2): most gathers miss L2 and
+    # reach HBM; 3001 rows of 21 uniform columns give partial last batches
+    # in every row
     w = wl.spmm_gemm_uniform(0x51A4 + K + L, 3001, 1 << 20, 21, K, L, name=f"spmm_gemm_wide_{K}")
     check(slnr, orc, w, "fused", True)
 

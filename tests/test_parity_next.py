@@ -169,7 +169,8 @@ def test_fused_is_deterministic_and_agrees_with_unfused(slnr, orc):
 
 
 def test_spmmh_gemm_gathered_matrices_larger_than_l2(slnr, orc):
-    # C and D have 2^20 rows of 128 floats: the Hadamard producers prefetch ahead
+    # C and D have 2^20 rows of 128 floats (1 GB, far more than L2): most of
+    # the Hadamard producers' gathers reach HBM
     r = wl.Rng(0x51A4 + 77)
     n, ncols, J, L = 2001, 1 << 20, 128, 64
     pos, crd = wl.uniform_csr_structure(r, n, ncols, 19)
