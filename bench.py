@@ -412,6 +412,8 @@ def main():
     ap.add_argument("--ref-gflop-per-expr", type=float, default=1.0)
     ap.add_argument("--expr", default="", help="only the expressions whose name contains this (profiling)")
     ap.add_argument("--scale", type=float, default=1.0, help="shrink the workloads (profiling captures)")
+    ap.add_argument("--sweep-k", default="", help="sweep: only these K (comma list; default all)")
+    ap.add_argument("--sweep-l", default="", help="sweep: only these L (comma list; default all)")
     ap.add_argument("--suite", choices=["main", "next", "sweep"], default="main",
                     help="main: the four benchmark expressions (the step); next: <SDDMM,SpMM,GEMM>, "
                          "<MTTKRP,GEMM>, <SpMMH,GEMM> at full size; sweep: <SpMM,GEMM> fused and unfused "
@@ -619,10 +621,12 @@ def run_sweep(args, rank, world, local):
     ws = slnr.Workspace(device=dev)
     stream = torch.cuda.current_stream()
     grid, t0 = [], time.time()
-    for K in SWEEP_DIMS:
+    ks = [int(x) for x in args.sweep_k.split(",")] if args.sweep_k else list(SWEEP_DIMS)
+    ls = [int(x) for x in args.sweep_l.split(",")] if args.sweep_l else list(SWEEP_DIMS)
+    for K in ks:
         rk = wl.Rng(seed ^ (K << 20))
         C = torch.from_numpy(wl.normal(rk, (n, K))).to(dev)
-        for L in SWEEP_DIMS:
+        for L in ls:
             rl = wl.Rng(seed ^ (K << 20) ^ (L << 8) ^ 1)
             D = torch.from_numpy(wl.normal(rl, (K, L))).to(dev)
             w = wl.Workload(f"spmm_gemm_rmat_k{K}_l{L}", "spmm_gemm", base.B, {}, {"K": K, "L": L})
@@ -655,7 +659,7 @@ def run_sweep(args, rank, world, local):
         "value": round(statistics.geometric_mean(r["unfused_over_fused"] for r in grid), 3), "unit": "x (geomean)",
         "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "n/a",
         "vs_baseline": None, "dtype": "f32 (tf32 tensor-core contractions allowed)", "data": "synthetic",
-        "config": {"workload": f"spmm_gemm R-MAT {n}x{n}, 16 nnz/row (seed {seed:#x}), K, L in {list(SWEEP_DIMS)}",
+        "config": {"workload": f"spmm_gemm R-MAT {n}x{n}, 16 nnz/row (seed {seed:#x}), K in {ks}, L in {ls}",
                    "l2": "flushed before every call", "timing": "median kernel time per call, CUDA events"},
         "best": {"K": best["K"], "L": best["L"], "unfused_over_fused": best["unfused_over_fused"]},
         "grid": grid, "seconds": round(time.time() - t0, 1),

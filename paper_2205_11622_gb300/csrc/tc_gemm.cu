@@ -348,16 +348,20 @@ __device__ __forceinline__ void st_stream(float* p, float4 x, uint64_t pol) {
 // most a warp), lane gl of the group holding the 4 columns [4 gl, 4 gl + 4)
 // as one float4; a warp holds G = 32 / GS groups.  A claim is IPC = G * R
 // consecutive items of an item tile, group g taking items g R .. g R + R - 1,
-// with R = min(GS, RB) (a lane of the group holds each item's record).  RB is
-// the short-wave width, or the long-item batch where every item runs on its
-// own (sampled rows: claims of 8 such items made the tiles of heavy-row
-// chunks at the head of the list twice as long).
+// with R = min(GS, RB) (a lane of the group holds each item's record).  A
+// claim's items run one after the other in each group, so the tiles of
+// heavy-row chunks at the head of the list take R items' time on the claims
+// of one tile; with narrow groups (many per warp) larger claims made those
+// tiles the kernel's tail.  Measured on the 2^20-row R-MAT graph: R = 1 at
+// K = 16 (0.55 -> 0.45 ms against R = 4), R = 2 at K = 32 (0.51 -> 0.42 ms
+// against R = 8), the short-wave width 8 at K >= 64, and 4 for sampled rows,
+// where every item runs on its own (8 doubled the heavy tiles' length).
 template <int K, bool SEQ>
 struct ProdLayout {
   static constexpr int VPL = K > 128 ? 8 : 4;  // a group is at most a warp
   static constexpr int GS = K / VPL;
   static constexpr int G = 32 / GS;
-  static constexpr int RB = SEQ ? kBatch : kShortBatch;
+  static constexpr int RB = G >= 8 ? 1 : G == 4 ? 2 : SEQ ? kBatch : kShortBatch;
   static constexpr int R = GS < RB ? GS : RB;
   static constexpr int IPC = G * R;
   static_assert(GS >= 1 && GS <= 32 && 32 % GS == 0, "a group is a power-of-two part of a warp");
