@@ -472,9 +472,13 @@ def main():
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     flush_buf = torch.empty(max(2 * l2, 64 << 20), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
-    slnr.timing_enable(True)
 
-    def one_step(record):
+    def one_step(hook):
+        """One call of every expression (L2 flushed before each); with hook, the
+        library's per-launch event hook is on and its kernel times are read
+        back.  The timed steps run without it: its event records sit between
+        the launches."""
+        slnr.timing_enable(hook)
         per_expr, per_kernel, launches = [], [], 0
         for i in range(len(ws)):
             flush_buf.fill_(i & 0xFF)
@@ -484,9 +488,10 @@ def main():
             b.record(stream)
             b.synchronize()
             per_expr.append(a.elapsed_time(b))
-            kt = slnr.timing_read()
+            kt = slnr.timing_read() if hook else []
             per_kernel.append(kt)
             launches += len(kt)
+        slnr.timing_enable(False)
         return per_expr, per_kernel, launches
 
     for _ in range(args.warmup):
@@ -504,18 +509,24 @@ def main():
     time.sleep(0.5)
     torch.cuda.synchronize()
     expr_ms = [[] for _ in ws]
-    kern_ms = [dict() for _ in ws]
-    gpu_launches = 0
     for _ in range(args.steps):
-        pe, pk, nl = one_step(True)
-        gpu_launches += nl
+        pe, _, _ = one_step(False)
         for i in range(len(ws)):
             expr_ms[i].append(pe[i])
-            for name, ms in pk[i]:
-                kern_ms[i][name] = kern_ms[i].get(name, 0.0) + ms
     torch.cuda.synchronize()
     time.sleep(0.3)
     clocks.stop()
+    # the kernel breakdown (and the launch count, the same in every step) from
+    # as many steps again with the hook on, outside the timed region
+    kern_ms = [dict() for _ in ws]
+    launches_per_step = 0
+    for _ in range(args.steps):
+        _, pk, nl = one_step(True)
+        launches_per_step = nl
+        for i in range(len(ws)):
+            for name, ms in pk[i]:
+                kern_ms[i][name] = kern_ms[i].get(name, 0.0) + ms
+    gpu_launches = launches_per_step * args.steps
     mean_ms = [statistics.mean(x) for x in expr_ms]
     total_flops = sum(flops)
     step_ms, value = job_throughput(sum(mean_ms), total_flops, world, pg, dev)
@@ -689,7 +700,11 @@ def config1_latency(torch, slnr, dev, args, allow_tf32, flush_buf, stream):
         b.synchronize()
         if it >= args.warmup:
             ts.append(a.elapsed_time(b))
+    slnr.timing_enable(True)  # one more call for the kernel breakdown
+    flush_buf.fill_(0)
+    slnr.run(w.op, B, dense, out=out, variant=args.variant, allow_tf32=allow_tf32, workspace=ws)
     kt = slnr.timing_read()
+    slnr.timing_enable(False)
     ms = statistics.mean(ts)
     return {"name": w.name, "entry": {
         "ms": round(ms, 4), "gflops": round(useful_flops(w) / (ms / 1e3) / 1e9, 2), "min_bytes": min_bytes(w),

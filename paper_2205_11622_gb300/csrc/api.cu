@@ -705,13 +705,7 @@ slnr_status slnr_spttm_ttm(const slnr_csf3* B, const float* C, int32_t L, const 
   SLNR_CHECK(begin(ws, s, opts->validate != 0,
                    [&](WsHeader* h) { return launch_validate_csf(*B, h, s); }));
   // A's two compressed levels are B's (the (i,j) pattern is unchanged)
-  SLNR_CUDA(cudaMemcpyAsync(A_pos1, B->pos1, 2 * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
-  SLNR_CUDA(cudaMemcpyAsync(A_pos2, B->pos2, ((size_t)B->nslices + 1) * sizeof(int32_t),
-                            cudaMemcpyDeviceToDevice, s));
-  if (B->nslices > 0)
-    SLNR_CUDA(cudaMemcpyAsync(A_crd1, B->crd1, (size_t)B->nslices * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
-  if (B->nfibers > 0)
-    SLNR_CUDA(cudaMemcpyAsync(A_crd2, B->crd2, (size_t)B->nfibers * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+  SLNR_LAUNCH("copy_levels", launch_copy_levels(*B, A_pos1, A_crd1, A_pos2, A_crd2, s));
   if (B->nfibers == 0) return SLNR_OK;
   const CsrView fv = fiber_view(B);
   const bool tc = use_tc(opts, L, M);

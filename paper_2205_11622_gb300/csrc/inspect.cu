@@ -107,6 +107,27 @@ __global__ void k_unit_ranges(const WsHeader* __restrict__ hdr, int max_units, c
   }
 }
 
+// A's compressed levels as copies of B's (<SpTTM,SpTTM>: the (i,j) pattern is
+// unchanged) in one launch: pos1 (2), pos2 (nslices + 1) and crd1 (nslices)
+// in a grid-stride pass over their concatenation, then crd2 (nfibers, the
+// bulk) in 16-byte pieces where both arrays are 16-byte aligned.
+__global__ void k_copy_levels(const int32_t* __restrict__ pos1, const int32_t* __restrict__ pos2,
+                              const int32_t* __restrict__ crd1, const int32_t* __restrict__ crd2, int32_t* a_pos1,
+                              int32_t* a_pos2, int32_t* a_crd1, int32_t* a_crd2, int nslices, int nfibers,
+                              bool vec) {
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t n0 = 2, n1 = n0 + nslices + 1, n2 = n1 + nslices;
+  for (int64_t i = tid; i < n2; i += stride) {
+    if (i < n0) a_pos1[i] = pos1[i];
+    else if (i < n1) a_pos2[i - n0] = pos2[i - n0];
+    else a_crd1[i - n1] = crd1[i - n1];
+  }
+  const int64_t n4 = vec ? nfibers / 4 : 0;
+  for (int64_t i = tid; i < n4; i += stride)
+    reinterpret_cast<int4*>(a_crd2)[i] = __ldg(reinterpret_cast<const int4*>(crd2) + i);
+  for (int64_t i = 4 * n4 + tid; i < nfibers; i += stride) a_crd2[i] = crd2[i];
+}
+
 // One thread per parent: checks its position range and the order and range of
 // its children's coordinates.  Ranges are clamped so a malformed array never
 // leads to an out-of-bounds read.
@@ -173,6 +194,18 @@ cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStrea
                                                                      plan.slice_units, plan.units, plan.max_units);
   k_unit_ranges<<<grid_for(plan.max_units, 256), 256, 0, s>>>(plan.hdr, plan.max_units, B.pos2, B.pos3,
                                                                plan.slice_units, plan.units);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_copy_levels(const slnr_csf3& B, int32_t* A_pos1, int32_t* A_crd1, int32_t* A_pos2,
+                               int32_t* A_crd2, cudaStream_t s) {
+  const bool vec = (reinterpret_cast<uintptr_t>(B.crd2) & 15u) == 0 && (reinterpret_cast<uintptr_t>(A_crd2) & 15u) == 0;
+  const int64_t n = 2 * (int64_t)B.nslices + 3 + (vec ? B.nfibers / 4 : B.nfibers);
+  const int64_t cap = (int64_t)device_sm_count() * 8;
+  int64_t grid = (n + 255) / 256;
+  if (grid > cap) grid = cap;
+  k_copy_levels<<<(unsigned)grid, 256, 0, s>>>(B.pos1, B.pos2, B.crd1, B.crd2, A_pos1, A_pos2, A_crd1, A_crd2,
+                                               B.nslices, B.nfibers, vec);
   return cudaGetLastError();
 }
 

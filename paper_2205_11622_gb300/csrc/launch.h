@@ -72,6 +72,9 @@ cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_
 cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s);
 cudaError_t launch_validate_csr(const slnr_csr& B, WsHeader* hdr, cudaStream_t s);
 cudaError_t launch_validate_csf(const slnr_csf3& B, WsHeader* hdr, cudaStream_t s);
+// A's levels pos1, crd1, pos2, crd2 copied from B's in one launch
+cudaError_t launch_copy_levels(const slnr_csf3& B, int32_t* A_pos1, int32_t* A_crd1, int32_t* A_pos2,
+                               int32_t* A_crd2, cudaStream_t s);
 
 // spmm.cu -- out[r,:] = sum_p vals[p] X[crd[p],:] (width W), and the heavy-row machinery
 // (with X2 not NULL the gathered row is X[k,:] .* X2[k,:], the <SpMMH,GEMM> producer)
