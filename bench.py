@@ -488,9 +488,8 @@ def main():
             b.record(stream)
             b.synchronize()
             per_expr.append(a.elapsed_time(b))
-            kt = slnr.timing_read() if hook else []
-            per_kernel.append(kt)
-            launches += len(kt)
+            per_kernel.append(slnr.timing_read() if hook else [])
+            launches += slnr.timing_launches()  # this library's kernels in the call
         slnr.timing_enable(False)
         return per_expr, per_kernel, launches
 
@@ -509,24 +508,23 @@ def main():
     time.sleep(0.5)
     torch.cuda.synchronize()
     expr_ms = [[] for _ in ws]
+    gpu_launches = 0
     for _ in range(args.steps):
-        pe, _, _ = one_step(False)
+        pe, _, nl = one_step(False)
+        gpu_launches += nl
         for i in range(len(ws)):
             expr_ms[i].append(pe[i])
     torch.cuda.synchronize()
     time.sleep(0.3)
     clocks.stop()
-    # the kernel breakdown (and the launch count, the same in every step) from
-    # as many steps again with the hook on, outside the timed region
+    # the per-phase breakdown from as many steps again with the hook on,
+    # outside the timed region
     kern_ms = [dict() for _ in ws]
-    launches_per_step = 0
     for _ in range(args.steps):
-        _, pk, nl = one_step(True)
-        launches_per_step = nl
+        _, pk, _ = one_step(True)
         for i in range(len(ws)):
             for name, ms in pk[i]:
                 kern_ms[i][name] = kern_ms[i].get(name, 0.0) + ms
-    gpu_launches = launches_per_step * args.steps
     mean_ms = [statistics.mean(x) for x in expr_ms]
     total_flops = sum(flops)
     step_ms, value = job_throughput(sum(mean_ms), total_flops, world, pg, dev)

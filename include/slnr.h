@@ -232,15 +232,20 @@ slnr_status slnr_sddmm_spmm_noalloc(const slnr_csr *B, const float *C, const flo
 
 /* ---- per-launch timing (instrumentation) --------------------------------
  * With timing enabled, each call on the calling thread records a CUDA event on
- * opts->stream before each of its kernel launches and one after the last, so
- * launch i's device duration is the time between events i and i+1.  A call
- * overwrites the previous call's record.  Reading a duration waits for the
- * call's last event.  Costs one event record per launch; off by default. */
+ * opts->stream before each of its phases (a named step of one or two kernel
+ * launches) and one after the last, so phase i's device duration is the time
+ * between events i and i+1.  A call overwrites the previous call's record.
+ * Reading a duration waits for the call's last event.  Costs one event record
+ * per phase; off by default. */
 slnr_status slnr_timing_enable(int32_t on);
-/* Kernel launches recorded by the calling thread's last call (0 if timing is off). */
+/* Phases recorded by the calling thread's last call (0 if timing is off). */
 int32_t slnr_timing_count(void);
-/* Name of launch i of the last call and its device time in milliseconds. */
+/* Name of phase i of the last call and its device time in milliseconds. */
 slnr_status slnr_timing_get(int32_t i, const char **name, float *ms);
+/* Kernel launches of the calling thread's last call (or of the call in
+ * progress), counted whether timing is on or not.  Memsets and copies the
+ * call enqueues are not kernels of this library and are not counted. */
+int32_t slnr_timing_launches(void);
 
 /* ---- bounded device-side waits ------------------------------------------
  * Every spin of the tensor-core kernels (on an mbarrier, a shared counter or

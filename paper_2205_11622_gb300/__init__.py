@@ -74,6 +74,7 @@ SIGNATURES = {
     "slnr_set_wait_limit": ([ctypes.c_int64], ctypes.c_int),
     "slnr_peak_ffma": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "slnr_peak_tf32": ([_P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+    "slnr_timing_launches": ([], ctypes.c_int32),
     "slnr_peak_gather": ([_P, ctypes.c_int64, ctypes.c_int, _P, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "slnr_timing_enable": ([_I32], ctypes.c_int),
     "slnr_timing_count": ([], ctypes.c_int32),
@@ -149,6 +150,11 @@ def peaks(stream=None, gather_width=None):
             out[key] = v.value
             del table
     return out
+
+
+def timing_launches():
+    """Kernel launches of the calling thread's last call (slnr_timing_launches)."""
+    return int(lib().slnr_timing_launches())
 
 
 def timing_read():

@@ -33,8 +33,12 @@ struct Timing {
   cudaEvent_t ev[kMaxTimed + 1] = {};
 };
 thread_local Timing g_timing;
+thread_local int32_t g_launches = 0;  // kernel launches of this thread's current call
 
-void timing_begin() { g_timing.n = 0; }
+void timing_begin() {
+  g_timing.n = 0;
+  g_launches = 0;
+}
 
 void timing_mark(const char* name, cudaStream_t s) {
   if (!g_timing.on || g_timing.n >= kMaxTimed) return;
@@ -399,6 +403,8 @@ void slnr::set_last_error(const char* msg) { snprintf(g_last_error, sizeof(g_las
 
 long long slnr::wait_limit_cycles() { return g_wait_limit > 0 ? g_wait_limit : kWaitCycles; }
 
+void slnr::note_launch() { ++g_launches; }
+
 // ===========================================================================
 
 extern "C" {
@@ -462,6 +468,8 @@ slnr_status slnr_timing_enable(int32_t on) {
 }
 
 int32_t slnr_timing_count(void) { return g_timing.on ? g_timing.n : 0; }
+
+int32_t slnr_timing_launches(void) { return g_launches; }
 
 slnr_status slnr_timing_get(int32_t i, const char** name, float* ms) {
   if (!g_timing.on || i < 0 || i >= g_timing.n) return fail(SLNR_ERR_SHAPE, "no timed launch %d", (int)i);

@@ -166,12 +166,12 @@ cudaError_t launch_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* 
           if (C2 == nullptr) {
             cudaError_t e = set_smem(k_spmm_gemm_rows<KC, LC, false>, smem);
             if (e != cudaSuccess) return e;
-            k_spmm_gemm_rows<KC, LC, false><<<(unsigned)ctas, 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C,
+            k_spmm_gemm_rows<KC, LC, false><<<SLNR_COUNTED((unsigned)ctas), 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C,
                                                                                nullptr, D, A);
           } else {
             cudaError_t e = set_smem(k_spmm_gemm_rows<KC, LC, true>, smem);
             if (e != cudaSuccess) return e;
-            k_spmm_gemm_rows<KC, LC, true><<<(unsigned)ctas, 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2,
+            k_spmm_gemm_rows<KC, LC, true><<<SLNR_COUNTED((unsigned)ctas), 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2,
                                                                               D, A);
           }
         }
@@ -185,12 +185,12 @@ cudaError_t launch_spmm_gemm_tiles(int K, int L, const CsrView& B, const float* 
     if (C2 == nullptr) {
       cudaError_t e = set_smem(k_spmm_gemm_tiles<KC, false>, smem);
       if (e != cudaSuccess) return e;
-      k_spmm_gemm_tiles<KC, false><<<(unsigned)grid, 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, nullptr, D,
+      k_spmm_gemm_tiles<KC, false><<<SLNR_COUNTED((unsigned)grid), 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, nullptr, D,
                                                                      L, A);
     } else {
       cudaError_t e = set_smem(k_spmm_gemm_tiles<KC, true>, smem);
       if (e != cudaSuccess) return e;
-      k_spmm_gemm_tiles<KC, true><<<(unsigned)grid, 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2, D, L,
+      k_spmm_gemm_tiles<KC, true><<<SLNR_COUNTED((unsigned)grid), 256, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2, D, L,
                                                                     A);
     }
   });
@@ -206,7 +206,7 @@ cudaError_t launch_dense_gemm(int64_t M, int K, int L, const float* T, const flo
   SLNR_WIDTH_SWITCH(K, KC, {
     cudaError_t e = set_smem(k_dense_gemm<KC>, smem);
     if (e != cudaSuccess) return e;
-    k_dense_gemm<KC><<<(unsigned)grid, 256, smem, s>>>(M, T, D, L, A);
+    k_dense_gemm<KC><<<SLNR_COUNTED((unsigned)grid), 256, smem, s>>>(M, T, D, L, A);
   });
   return cudaGetLastError();
 }

@@ -183,16 +183,16 @@ inline int grid_for(int64_t n, int block) {
 
 cudaError_t launch_classify(const CsrView& B, const SplitPlan& plan, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
-  k_classify<<<grid_for(B.nrows, 256), 256, 0, s>>>(B.nrows, B.pos, plan.hdr, plan.heavy, plan.chunks,
+  k_classify<<<SLNR_COUNTED(grid_for(B.nrows, 256)), 256, 0, s>>>(B.nrows, B.pos, plan.hdr, plan.heavy, plan.chunks,
                                                     plan.max_heavy, plan.max_chunks);
   return cudaGetLastError();
 }
 
 cudaError_t launch_csf_units(const slnr_csf3& B, const UnitPlan& plan, cudaStream_t s) {
   if (B.nslices <= 0) return cudaSuccess;
-  k_csf_units<<<grid_for((int64_t)B.nslices * 32, 256), 256, 0, s>>>(B.nslices, B.pos2, B.pos3, plan.hdr,
+  k_csf_units<<<SLNR_COUNTED(grid_for((int64_t)B.nslices * 32, 256)), 256, 0, s>>>(B.nslices, B.pos2, B.pos3, plan.hdr,
                                                                      plan.slice_units, plan.units, plan.max_units);
-  k_unit_ranges<<<grid_for(plan.max_units, 256), 256, 0, s>>>(plan.hdr, plan.max_units, B.pos2, B.pos3,
+  k_unit_ranges<<<SLNR_COUNTED(grid_for(plan.max_units, 256)), 256, 0, s>>>(plan.hdr, plan.max_units, B.pos2, B.pos3,
                                                                plan.slice_units, plan.units);
   return cudaGetLastError();
 }
@@ -204,19 +204,19 @@ cudaError_t launch_copy_levels(const slnr_csf3& B, int32_t* A_pos1, int32_t* A_c
   const int64_t cap = (int64_t)device_sm_count() * 8;
   int64_t grid = (n + 255) / 256;
   if (grid > cap) grid = cap;
-  k_copy_levels<<<(unsigned)grid, 256, 0, s>>>(B.pos1, B.pos2, B.crd1, B.crd2, A_pos1, A_pos2, A_crd1, A_crd2,
+  k_copy_levels<<<SLNR_COUNTED((unsigned)grid), 256, 0, s>>>(B.pos1, B.pos2, B.crd1, B.crd2, A_pos1, A_pos2, A_crd1, A_crd2,
                                                B.nslices, B.nfibers, vec);
   return cudaGetLastError();
 }
 
 cudaError_t launch_validate_csr(const slnr_csr& B, WsHeader* hdr, cudaStream_t s) {
-  k_validate_csr<<<grid_for(B.nrows > 0 ? B.nrows : 1, 256), 256, 0, s>>>(B, hdr);
+  k_validate_csr<<<SLNR_COUNTED(grid_for(B.nrows > 0 ? B.nrows : 1, 256)), 256, 0, s>>>(B, hdr);
   return cudaGetLastError();
 }
 
 cudaError_t launch_validate_csf(const slnr_csf3& B, WsHeader* hdr, cudaStream_t s) {
   const int64_t n = B.nfibers > B.nslices ? B.nfibers : B.nslices;
-  k_validate_csf<<<grid_for(n > 0 ? n : 1, 256), 256, 0, s>>>(B, hdr);
+  k_validate_csf<<<SLNR_COUNTED(grid_for(n > 0 ? n : 1, 256)), 256, 0, s>>>(B, hdr);
   return cudaGetLastError();
 }
 

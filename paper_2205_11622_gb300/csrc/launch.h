@@ -10,6 +10,11 @@
 
 namespace slnr {
 
+// Counts the calling thread's kernel launches: every launch's grid argument is
+// wrapped in SLNR_COUNTED; a call's count starts at 0 (slnr_timing_launches).
+void note_launch();
+#define SLNR_COUNTED(grid) (::slnr::note_launch(), (grid))
+
 // A CSR-shaped view: rows with positions pos[nrows+1], coordinates crd and
 // values vals.  CSF fibers are viewed this way too (rows = fibers,
 // pos = pos3, crd = crd3).

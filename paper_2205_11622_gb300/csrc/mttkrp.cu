@@ -389,7 +389,7 @@ cudaError_t launch_mttkrp_units(int L, const slnr_csf3& B, const float* C, const
   SLNR_WIDTH_SWITCH(L, W, {
     int ctas = grid_units(plan.max_units);  // as many as stay resident: warps take units dynamically
     if (ctas > device_sm_count() * SLNR_MTTKRP_MIN_CTAS) ctas = device_sm_count() * SLNR_MTTKRP_MIN_CTAS;
-    k_mttkrp_units<W><<<ctas, 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units,
+    k_mttkrp_units<W><<<SLNR_COUNTED(ctas), 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units,
                                                                  plan.max_units, B.pos2, B.crd2, B.pos3,
                                                                  B.crd3, B.vals, C, D, plan.partial);
   });
@@ -400,7 +400,7 @@ cudaError_t launch_mttkrp_stage2_units(int L, const slnr_csf3& B, const float* T
                                        const UnitPlan& plan, cudaStream_t s) {
   if (plan.max_units <= 0 || B.nslices <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_mttkrp_stage2_units<W><<<grid_units(plan.max_units), 256, 0, s>>>(
+    k_mttkrp_stage2_units<W><<<SLNR_COUNTED(grid_units(plan.max_units)), 256, 0, s>>>(
         plan.hdr, plan.units, plan.slice_units, plan.max_units, B.pos2, B.crd2, B.pos3, T, C, plan.partial);
   });
   return cudaGetLastError();
@@ -418,9 +418,9 @@ cudaError_t launch_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& pla
   SLNR_WIDTH_SWITCH(L, W, {
     int64_t pgrid = ceil_div(plan.max_units, 32 * 8);  // a warp per 32 units
     if (pgrid > (int64_t)device_sm_count() * 32) pgrid = (int64_t)device_sm_count() * 32;
-    k_mttkrp_parts<W><<<(unsigned)pgrid, 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units, plan.max_units,
+    k_mttkrp_parts<W><<<SLNR_COUNTED((unsigned)pgrid), 256, 0, s>>>(plan.hdr, plan.units, plan.slice_units, plan.max_units,
                                                       plan.partial, plan.part_sums);
-    k_mttkrp_combine<W><<<(unsigned)grid, 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial,
+    k_mttkrp_combine<W><<<SLNR_COUNTED((unsigned)grid), 256, 0, s>>>(B.nslices, B.crd1, plan.slice_units, plan.partial,
                                                        plan.part_sums, E, M, A);
   });
   return cudaGetLastError();

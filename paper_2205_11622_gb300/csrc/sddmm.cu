@@ -335,7 +335,7 @@ cudaError_t launch_sddmm_spmm_rows(const CsrView& B, const float* C, const float
   const int64_t cap = (int64_t)device_sm_count() * SLNR_SDDMM_MIN_CTAS;
   if (ctas > cap) ctas = cap;
   SLNR_WIDTH_SWITCH(WM, W, {
-    k_sddmm_spmm_rows<W><<<(unsigned)ctas, 256, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A,
+    k_sddmm_spmm_rows<W><<<SLNR_COUNTED((unsigned)ctas), 256, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, C, D, L, E, K, A,
                                                          plan.chunks, plan.max_chunks, plan.partial);
   });
   return cudaGetLastError();
@@ -346,7 +346,7 @@ cudaError_t launch_sddmm_spmm_chunks(const CsrView& B, const float* C, const flo
   if (plan.max_chunks <= 0) return cudaSuccess;
   const int WM = L > K ? L : K;
   SLNR_WIDTH_SWITCH(WM, W, {
-    k_sddmm_spmm_chunks<W><<<grid_rows(plan.max_chunks), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks,
+    k_sddmm_spmm_chunks<W><<<SLNR_COUNTED(grid_rows(plan.max_chunks)), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks,
                                                                       B.crd, B.vals, C, D, L, E, K,
                                                                       plan.partial);
   });
@@ -364,7 +364,7 @@ cudaError_t launch_sddmm_spmm_gemm_tiles(const CsrView& B, const float* C, const
       if (LC <= WMC) {
         cudaError_t e = set_smem(k_sddmm_spmm_gemm_tiles<WMC, LC <= WMC ? LC : WMC>, smem);
         if (e != cudaSuccess) return e;
-        k_sddmm_spmm_gemm_tiles<WMC, LC <= WMC ? LC : WMC><<<(unsigned)grid, 256, smem, s>>>(
+        k_sddmm_spmm_gemm_tiles<WMC, LC <= WMC ? LC : WMC><<<SLNR_COUNTED((unsigned)grid), 256, smem, s>>>(
             B.nrows, B.pos, B.crd, B.vals, C, D, K, F, W, M, A);
       }
     });
@@ -376,7 +376,7 @@ cudaError_t launch_sddmm_rows(const CsrView& B, const float* C, const float* D, 
                               cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_sddmm_rows<W><<<grid_rows(B.nrows), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, C, D, Y);
+    k_sddmm_rows<W><<<SLNR_COUNTED(grid_rows(B.nrows)), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, C, D, Y);
   });
   return cudaGetLastError();
 }
@@ -385,7 +385,7 @@ cudaError_t launch_sddmm_chunks(const CsrView& B, const float* C, const float* D
                                 const SplitPlan& plan, cudaStream_t s) {
   if (plan.max_chunks <= 0) return cudaSuccess;
   SLNR_WIDTH_SWITCH(L, W, {
-    k_sddmm_chunks<W><<<grid_rows(plan.max_chunks), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks,
+    k_sddmm_chunks<W><<<SLNR_COUNTED(grid_rows(plan.max_chunks)), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks,
                                                                  B.crd, B.vals, C, D, Y);
   });
   return cudaGetLastError();

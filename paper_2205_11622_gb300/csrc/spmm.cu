@@ -54,27 +54,29 @@ __global__ void __launch_bounds__(256) k_spmm_chunks(const WsHeader* __restrict_
 }
 
 // Heavy rows with at most this many partials are summed by one warp when no D
-// follows (k_combine_rows); longer ones by a CTA (k_combine).
+// follows, longer ones by a CTA, both in one launch (k_combine_rows); with D
+// every row by a CTA (k_combine).
 constexpr int kWarpCombine = 16;
 
 // One CTA per heavy row: the row's partials (width W) are summed by
 // kRowLanes lanes each taking every kRowLanes-th partial, then by a fixed
 // pairwise tree, so the result does not depend on scheduling and long rows
 // keep a short rounding chain.  With D, the sum t (length W = K) is then
-// multiplied by D (K x L): out[row, l] = sum_k t[k] D[k, l].
+// multiplied by D (K x L): out[row, l] = sum_k t[k] D[k, l].  Without D, rows
+// of at most kWarpCombine partials are left to the warps of k_combine_rows.
+// The CTA's share: heavy rows first, first + stride, ... (block-uniform).
 template <int W>
-__global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hdr,
-                                                 const HeavyRow* __restrict__ heavy, int max_heavy,
-                                                 const float* __restrict__ partial,
-                                                 const float* __restrict__ D, int L,
-                                                 float* __restrict__ out) {
+__device__ __forceinline__ void combine_cta(const WsHeader* __restrict__ hdr, const HeavyRow* __restrict__ heavy,
+                                            int max_heavy, const float* __restrict__ partial,
+                                            const float* __restrict__ D, int L, float* __restrict__ out, int first,
+                                            int stride) {
   constexpr int NC = W / 4;                 // float4 columns
   constexpr int NR = 256 / NC;              // lanes along the partials
   __shared__ float4 red[256];
   __shared__ float t[W];
   const int n = min(hdr->n_heavy, max_heavy);
   const int c4 = threadIdx.x % NC, rl = threadIdx.x / NC;
-  for (int h = blockIdx.x; h < n; h += gridDim.x) {
+  for (int h = first; h < n; h += stride) {
     const HeavyRow hr = heavy[h];
     if (D == nullptr && hr.count <= kWarpCombine) continue;  // k_combine_rows writes it (block-uniform)
     float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -114,20 +116,27 @@ __global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hd
   }
 }
 
+template <int W>
+__global__ void __launch_bounds__(256) k_combine(const WsHeader* __restrict__ hdr,
+                                                 const HeavyRow* __restrict__ heavy, int max_heavy,
+                                                 const float* __restrict__ partial,
+                                                 const float* __restrict__ D, int L,
+                                                 float* __restrict__ out) {
+  combine_cta<W>(hdr, heavy, max_heavy, partial, D, L, out, blockIdx.x, gridDim.x);
+}
+
 // Without D, rows of at most kWarpCombine partials: a warp per heavy row
 // (grid-stride), lane l holding the columns [VPL l, VPL l + VPL); the row's
 // partials are added in their order (four loads in flight) and the sum
 // written.  Deterministic: the order is fixed.  Rows with more partials go to
-// k_combine, whose lanes split them.
+// the CTAs of combine_cta, whose lanes split them.
 template <int W>
-__global__ void __launch_bounds__(256) k_combine_rows(const WsHeader* __restrict__ hdr,
-                                                      const HeavyRow* __restrict__ heavy, int max_heavy,
-                                                      const float* __restrict__ partial, float* __restrict__ out) {
+__device__ __forceinline__ void combine_warps(const WsHeader* __restrict__ hdr, const HeavyRow* __restrict__ heavy,
+                                              int max_heavy, const float* __restrict__ partial,
+                                              float* __restrict__ out, int64_t warp, int64_t nwarps) {
   using RL = RowLanes<W>;
   const int n = min(hdr->n_heavy, max_heavy);
   const int lane = threadIdx.x & 31, grp = lane / RL::GS, col = (lane % RL::GS) * RL::VPL;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t h = warp * RL::GPW + grp; h < n; h += nwarps * RL::GPW) {
     const HeavyRow hr = heavy[h];
     if (hr.count > kWarpCombine) continue;
@@ -153,6 +162,23 @@ __global__ void __launch_bounds__(256) k_combine_rows(const WsHeader* __restrict
   }
 }
 
+// Without D, both kinds of heavy row in one launch: the first `nbig` CTAs
+// take the rows of more than kWarpCombine partials (a CTA each, as
+// k_combine), the other CTAs' warps the rest (a warp each, in order).
+template <int W>
+__global__ void __launch_bounds__(256) k_combine_rows(const WsHeader* __restrict__ hdr,
+                                                      const HeavyRow* __restrict__ heavy, int max_heavy,
+                                                      const float* __restrict__ partial, float* __restrict__ out,
+                                                      int nbig) {
+  if ((int)blockIdx.x < nbig) {
+    combine_cta<W>(hdr, heavy, max_heavy, partial, nullptr, 0, out, blockIdx.x, nbig);
+    return;
+  }
+  const int64_t warp = ((int64_t)(blockIdx.x - nbig) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)(gridDim.x - nbig) * blockDim.x) >> 5;
+  combine_warps<W>(hdr, heavy, max_heavy, partial, out, warp, nwarps);
+}
+
 inline int grid_warps(int64_t items_per_warp_round, int64_t n) {
   // enough CTAs of 8 warps to cover n items (items_per_warp_round per warp),
   // capped at 32 CTAs per SM; grid-stride loops cover the rest
@@ -171,9 +197,9 @@ cudaError_t launch_spmm_rows(int W, const CsrView& B, const float* X, float* out
   SLNR_WIDTH_SWITCH(W, WC, {
     const int grid = grid_warps(RowLanes<WC>::GPW, B.nrows);
     if (X2 == nullptr)
-      k_spmm_rows<WC, false><<<grid, 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, nullptr, out);
+      k_spmm_rows<WC, false><<<SLNR_COUNTED(grid), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, nullptr, out);
     else
-      k_spmm_rows<WC, true><<<grid, 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, X2, out);
+      k_spmm_rows<WC, true><<<SLNR_COUNTED(grid), 256, 0, s>>>(B.nrows, B.pos, B.crd, B.vals, X, X2, out);
   });
   return cudaGetLastError();
 }
@@ -184,10 +210,10 @@ cudaError_t launch_spmm_chunks(int W, const CsrView& B, const float* X, const Sp
   SLNR_WIDTH_SWITCH(W, WC, {
     const int grid = grid_warps(RowLanes<WC>::GPW, plan.max_chunks);
     if (X2 == nullptr)
-      k_spmm_chunks<WC, false><<<grid, 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X,
+      k_spmm_chunks<WC, false><<<SLNR_COUNTED(grid), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X,
                                                      nullptr, plan.partial);
     else
-      k_spmm_chunks<WC, true><<<grid, 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X, X2,
+      k_spmm_chunks<WC, true><<<SLNR_COUNTED(grid), 256, 0, s>>>(plan.hdr, plan.chunks, plan.max_chunks, B.crd, B.vals, X, X2,
                                                     plan.partial);
   });
   return cudaGetLastError();
@@ -199,16 +225,16 @@ cudaError_t launch_combine(int W, const SplitPlan& plan, const float* D, int L, 
   int grid = plan.max_heavy;
   const int cap = device_sm_count() * 8;
   if (grid > cap) grid = cap;
-  if (D == nullptr) {  // rows with few partials: a warp each; the rest below
+  if (D == nullptr) {  // rows with many partials a CTA each, the others a warp each, in one launch
+    const int nbig = device_sm_count() * 2 < grid ? device_sm_count() * 2 : grid;
     SLNR_WIDTH_SWITCH(W, WC, {
-      k_combine_rows<WC><<<grid_warps(RowLanes<WC>::GPW, plan.max_heavy), 256, 0, s>>>(
-          plan.hdr, plan.heavy, plan.max_heavy, plan.partial, out);
+      k_combine_rows<WC><<<SLNR_COUNTED(nbig + grid_warps(RowLanes<WC>::GPW, plan.max_heavy)), 256, 0, s>>>(
+          plan.hdr, plan.heavy, plan.max_heavy, plan.partial, out, nbig);
     });
-    const cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
   }
   SLNR_WIDTH_SWITCH(W, WC, {
-    k_combine<WC><<<grid, 256, 0, s>>>(plan.hdr, plan.heavy, plan.max_heavy, plan.partial, D, L, out);
+    k_combine<WC><<<SLNR_COUNTED(grid), 256, 0, s>>>(plan.hdr, plan.heavy, plan.max_heavy, plan.partial, D, L, out);
   });
   return cudaGetLastError();
 }

@@ -1058,7 +1058,7 @@ cudaError_t tc_dispatch(int K, int L, int64_t items_upper, WsHeader* hdr, const 
     if (grid > tl.grid_cap) grid = tl.grid_cap;                                                           \
     if (grid < 1) grid = 1;                                                                               \
     if ((e = cudaMemsetAsync(&hdr->next_tile, 0, sizeof(int), s)) != cudaSuccess) return e;               \
-    k_tc_gemm<KK, LL, MODE><<<(unsigned)grid, kTcThreads, tl.smem, s>>>(hdr, segs, max_segs, dense_rows,  \
+    k_tc_gemm<KK, LL, MODE><<<SLNR_COUNTED((unsigned)grid), kTcThreads, tl.smem, s>>>(hdr, segs, max_segs, dense_rows,  \
                                                                          crd, vals, X, X2, Cq, D, A,     \
                                                                          partial, wait);                 \
     return cudaGetLastError();                                                                            \
@@ -1090,14 +1090,14 @@ int seg_scan_blocks(int64_t nrows) { return (int)((nrows + kScanRows - 1) / kSca
 
 cudaError_t launch_seg_count(const CsrView& B, const SegPlan& plan, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
-  k_seg_count<<<seg_scan_blocks(B.nrows), kScanThreads, 0, s>>>(B.nrows, B.pos, plan.block_counts);
+  k_seg_count<<<SLNR_COUNTED(seg_scan_blocks(B.nrows)), kScanThreads, 0, s>>>(B.nrows, B.pos, plan.block_counts);
   return cudaGetLastError();
 }
 
 cudaError_t launch_seg_write(const CsrView& B, const SegPlan& plan, cudaStream_t s) {
   if (B.nrows <= 0) return cudaSuccess;
   const int nb = seg_scan_blocks(B.nrows);
-  k_seg_write<<<nb, kScanThreads, 0, s>>>(B.nrows, B.pos, plan.block_counts, nb, plan.hdr, plan.segs, plan.heavy,
+  k_seg_write<<<SLNR_COUNTED(nb), kScanThreads, 0, s>>>(B.nrows, B.pos, plan.block_counts, nb, plan.hdr, plan.segs, plan.heavy,
                                           plan.max_segs, plan.max_heavy, plan.max_chunks);
   return cudaGetLastError();
 }

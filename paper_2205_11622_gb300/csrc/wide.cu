@@ -550,10 +550,10 @@ cudaError_t launch_w_spmm(int W, const CsrView& B, const float* X, const float* 
   const unsigned grid = w_grid((int64_t)B.nrows + plan.max_chunks);
   SLNR_NCH_SWITCH(W, NC, {
     if (X2 == nullptr)
-      k_w_spmm<NC, false><<<grid, kWThreads, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, X, nullptr, W, out,
+      k_w_spmm<NC, false><<<SLNR_COUNTED(grid), kWThreads, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, X, nullptr, W, out,
                                                      plan.chunks, plan.max_chunks, plan.partial);
     else
-      k_w_spmm<NC, true><<<grid, kWThreads, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, X, X2, W, out,
+      k_w_spmm<NC, true><<<SLNR_COUNTED(grid), kWThreads, 0, s>>>(plan.hdr, B.nrows, B.pos, B.crd, B.vals, X, X2, W, out,
                                                     plan.chunks, plan.max_chunks, plan.partial);
   });
   return cudaGetLastError();
@@ -565,7 +565,7 @@ cudaError_t launch_w_combine(int W, const SplitPlan& plan, const float* D, int L
   SLNR_NCH_SWITCH(W, NC, {
     cudaError_t e = w_smem(k_w_combine<NC>, smem);
     if (e != cudaSuccess) return e;
-    k_w_combine<NC><<<w_grid(plan.max_heavy), kWThreads, smem, s>>>(plan.hdr, plan.heavy, plan.max_heavy,
+    k_w_combine<NC><<<SLNR_COUNTED(w_grid(plan.max_heavy)), kWThreads, smem, s>>>(plan.hdr, plan.heavy, plan.max_heavy,
                                                                      plan.partial, W, D, L, out);
   });
   return cudaGetLastError();
@@ -580,12 +580,12 @@ cudaError_t launch_w_spmm_gemm_tiles(int K, int L, const CsrView& B, const float
     if (C2 == nullptr) {
       cudaError_t e = w_smem(k_w_spmm_gemm_tiles<NC, false>, smem);
       if (e != cudaSuccess) return e;
-      k_w_spmm_gemm_tiles<NC, false><<<(unsigned)grid, kWThreads, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C,
+      k_w_spmm_gemm_tiles<NC, false><<<SLNR_COUNTED((unsigned)grid), kWThreads, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C,
                                                                              nullptr, K, D, L, A);
     } else {
       cudaError_t e = w_smem(k_w_spmm_gemm_tiles<NC, true>, smem);
       if (e != cudaSuccess) return e;
-      k_w_spmm_gemm_tiles<NC, true><<<(unsigned)grid, kWThreads, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2,
+      k_w_spmm_gemm_tiles<NC, true><<<SLNR_COUNTED((unsigned)grid), kWThreads, smem, s>>>(B.nrows, B.pos, B.crd, B.vals, C, C2,
                                                                             K, D, L, A);
     }
   });
@@ -597,7 +597,7 @@ cudaError_t launch_w_dense_gemm(int64_t M, int K, int L, const float* T, const f
   const size_t smem = wtile_smem(K);
   cudaError_t e = w_smem(k_w_dense_gemm, smem);
   if (e != cudaSuccess) return e;
-  k_w_dense_gemm<<<(unsigned)ceil_div(M, kWTileRows), kWThreads, smem, s>>>(M, T, K, D, L, A);
+  k_w_dense_gemm<<<SLNR_COUNTED((unsigned)ceil_div(M, kWTileRows)), kWThreads, smem, s>>>(M, T, K, D, L, A);
   return cudaGetLastError();
 }
 
@@ -609,7 +609,7 @@ cudaError_t launch_w_sddmm_spmm(const CsrView& B, const float* C, const float* D
   SLNR_NCH_SWITCH(wmax, NC, {
     cudaError_t e = w_smem(k_w_sddmm_spmm<NC>, smem);
     if (e != cudaSuccess) return e;
-    k_w_sddmm_spmm<NC><<<w_grid((int64_t)B.nrows + plan.max_chunks), kWThreads, smem, s>>>(
+    k_w_sddmm_spmm<NC><<<SLNR_COUNTED(w_grid((int64_t)B.nrows + plan.max_chunks)), kWThreads, smem, s>>>(
         plan.hdr, B.nrows, B.pos, B.crd, B.vals, C, D, Kd, E, Ko, A, plan.chunks, plan.max_chunks, plan.partial, Y);
   });
   return cudaGetLastError();
@@ -623,7 +623,7 @@ cudaError_t launch_w_sddmm_spmm_gemm_tiles(const CsrView& B, const float* C, con
   SLNR_NCH_SWITCH(wmax, NC, {
     cudaError_t e = w_smem(k_w_sddmm_spmm_gemm_tiles<NC>, smem);
     if (e != cudaSuccess) return e;
-    k_w_sddmm_spmm_gemm_tiles<NC><<<(unsigned)ceil_div(B.nrows, kWTileRows), kWThreads, smem, s>>>(
+    k_w_sddmm_spmm_gemm_tiles<NC><<<SLNR_COUNTED((unsigned)ceil_div(B.nrows, kWTileRows)), kWThreads, smem, s>>>(
         B.nrows, B.pos, B.crd, B.vals, C, D, K, F, L, W, M, A);
   });
   return cudaGetLastError();
@@ -635,10 +635,10 @@ cudaError_t launch_w_mttkrp_units(int L, const slnr_csf3& B, const float* C, con
   const unsigned grid = w_grid(plan.max_units);
   SLNR_NCH_SWITCH(L, NC, {
     if (T == nullptr)
-      k_w_mttkrp_units<NC, false><<<grid, kWThreads, 0, s>>>(plan.hdr, plan.units, plan.max_units, B.crd2, B.pos3,
+      k_w_mttkrp_units<NC, false><<<SLNR_COUNTED(grid), kWThreads, 0, s>>>(plan.hdr, plan.units, plan.max_units, B.crd2, B.pos3,
                                                              B.crd3, B.vals, C, D, nullptr, L, plan.partial);
     else
-      k_w_mttkrp_units<NC, true><<<grid, kWThreads, 0, s>>>(plan.hdr, plan.units, plan.max_units, B.crd2, B.pos3,
+      k_w_mttkrp_units<NC, true><<<SLNR_COUNTED(grid), kWThreads, 0, s>>>(plan.hdr, plan.units, plan.max_units, B.crd2, B.pos3,
                                                             B.crd3, B.vals, C, D, T, L, plan.partial);
   });
   return cudaGetLastError();
@@ -653,7 +653,7 @@ cudaError_t launch_w_mttkrp_combine(int L, const slnr_csf3& B, const UnitPlan& p
   SLNR_NCH_SWITCH(L, NC, {
     e = w_smem(k_w_mttkrp_combine<NC>, smem);
     if (e != cudaSuccess) return e;
-    k_w_mttkrp_combine<NC><<<w_grid(B.nslices), kWThreads, smem, s>>>(B.nslices, B.crd1, plan.slice_units,
+    k_w_mttkrp_combine<NC><<<SLNR_COUNTED(w_grid(B.nslices)), kWThreads, smem, s>>>(B.nslices, B.crd1, plan.slice_units,
                                                                         plan.partial, L, E, M, A);
   });
   return cudaGetLastError();

@@ -292,7 +292,10 @@ def test_fused_call_routing(slnr, orc, op, size):
     try:
         check(slnr, orc, w, "fused", True)
         names = [name for name, _ in slnr.timing_read()]
+        launches = slnr.timing_launches()
     finally:
         slnr.timing_enable(False)
     on_tc = any(name.startswith("tc_") for name in names)
     assert on_tc == (size == "large"), names
+    # every phase launches at least one kernel; none launches more than two
+    assert len(names) <= launches <= 2 * len(names), (names, launches)
