@@ -204,13 +204,17 @@ def gather_row_width(w) -> int:
     return v
 
 
+# sources whose code runs outside the measured calls: the peak kernels, the
+# entry point without a workspace, the perfect-loop-nest comparator
+OUTSIDE_MEASURED = ("peaks.cu", "noalloc.cu", "original.cu")
+
+
 def kernel_source_hash() -> str:
-    """Hash of the kernel sources that run inside the measured calls (the
-    peak-measuring kernels of peaks.cu run outside them)."""
+    """Hash of the kernel sources that run inside the measured calls."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2205_11622_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")) and name != "peaks.cu":
+        if name.endswith((".cu", ".cuh", ".h")) and name not in OUTSIDE_MEASURED:
             h.update(name.encode())
             h.update(open(os.path.join(csrc, name), "rb").read())
     return h.hexdigest()[:16]
@@ -414,6 +418,8 @@ def main():
     ap.add_argument("--scale", type=float, default=1.0, help="shrink the workloads (profiling captures)")
     ap.add_argument("--sweep-k", default="", help="sweep: only these K (comma list; default all)")
     ap.add_argument("--sweep-l", default="", help="sweep: only these L (comma list; default all)")
+    ap.add_argument("--original", action="store_true",
+                    help="sweep: also time the perfect loop nest (O(nnz K L); use with --scale, Fig. 8b)")
     ap.add_argument("--suite", choices=["main", "next", "sweep"], default="main",
                     help="main: the four benchmark expressions (the step); next: <SDDMM,SpMM,GEMM>, "
                          "<MTTKRP,GEMM>, <SpMMH,GEMM> at full size; sweep: <SpMM,GEMM> fused and unfused "
@@ -614,7 +620,9 @@ def run_sweep(args, rank, world, local):
     graph of the benchmark (16 nonzeros per row) for every inner-dimension
     pair K, L in SWEEP_DIMS, fused and unfused (TF32 allowed), kernel time per
     call (median, L2 flushed before each).  C (n x K) and D (K x L) are N(0,1)
-    from a seed derived from K and L; the graph is generated once."""
+    from a seed derived from K and L; the graph is generated once.  With
+    --original, also the perfect loop nest i, j, k, l (Fig. 8b's comparator,
+    O(nnz K L); 1 warm-up and up to 3 timed calls per cell)."""
     import torch
 
     import paper_2205_11622_gb300 as slnr
@@ -656,6 +664,19 @@ def run_sweep(args, rank, world, local):
                 res[f"{variant}_ms"] = round(statistics.median(ts), 4)
                 if slnr.device_flags() != 0:
                     raise SystemExit(f"device flags {slnr.device_flags():#x} at K={K}, L={L}, {variant}")
+            if args.original:  # the comparator: 1 warm-up, up to 3 timed calls
+                ts = []
+                for it in range(1 + min(3, args.steps)):
+                    flush.fill_(it & 0xFF)
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    slnr.spmm_gemm_original(B, C, D, out=out)
+                    b.record(stream)
+                    b.synchronize()
+                    if it >= 1:
+                        ts.append(a.elapsed_time(b))
+                res["original_ms"] = round(statistics.median(ts), 4)
+                res["original_over_fused"] = round(res["original_ms"] / res["fused_ms"], 2)
             res["unfused_over_fused"] = round(res["unfused_ms"] / res["fused_ms"], 3)
             res["fused_gflops"] = round(res["useful_flops"] / res["fused_ms"] / 1e6, 1)
             res["fused_hbm_frac"] = round(res["min_bytes"] / res["fused_ms"] / 1e6 / measured_peaks()[0], 4)
@@ -671,6 +692,8 @@ def run_sweep(args, rank, world, local):
         "config": {"workload": f"spmm_gemm R-MAT {n}x{n}, 16 nnz/row (seed {seed:#x}), K in {ks}, L in {ls}",
                    "l2": "flushed before every call", "timing": "median kernel time per call, CUDA events"},
         "best": {"K": best["K"], "L": best["L"], "unfused_over_fused": best["unfused_over_fused"]},
+        "original_over_fused_geomean": round(statistics.geometric_mean(r["original_over_fused"] for r in grid), 2)
+        if args.original else None,
         "grid": grid, "seconds": round(time.time() - t0, 1),
     }
     if rank == 0:

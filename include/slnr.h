@@ -220,8 +220,7 @@ slnr_status slnr_spmmh_gemm(const slnr_csr *B, const float *C, const float *D, i
  * nothing.  Sizes whose scratch would exceed 16 MiB (about 7 million nonzeros
  * at K = 64) return SLNR_ERR_UNSUPPORTED.  The first call on each device
  * looks up the array's device address (cudaGetSymbolAddress) with that device
- * current and keeps it; make that first call before any stream capture
- * begins.  A device reset (cudaDeviceReset) leaves the kept address stale:
+ * current and keeps it.  A device reset (cudaDeviceReset) leaves the kept address stale:
  * do not call this entry point on a device after resetting it.  All calls
  * share the one array: the call clears what must start at zero itself, and
  * calls whose work overlaps on the GPU (other streams, other host threads)
@@ -229,6 +228,19 @@ slnr_status slnr_spmmh_gemm(const slnr_csr *B, const float *C, const float *D, i
  * validate off and fp32 arithmetic. */
 slnr_status slnr_sddmm_spmm_noalloc(const slnr_csr *B, const float *C, const float *D, int32_t L,
                                     const float *E, int32_t K, float *A, void *stream);
+
+/* ---- comparator: <SpMM,GEMM> as the perfect loop nest ---------------------
+ * A(i,l) = sum_{j,k} B(i,j) C(j,k) D(k,l) evaluated with the loops i, j, k, l
+ * nested in that order and no temporary: the schedule without SparseLNR's
+ * transformation ("TACO Original" in Sec. 6), O(nnz K L) work.  It is the
+ * comparator of the inner-dimension case study (Sec. 6.3, Fig. 8b), not a
+ * variant of the fused path.  Arguments and layout as slnr_spmm_gemm (B, K
+ * and L are checked the same way; C, D, A device pointers, A written
+ * whole); fp32 arithmetic, one chain per output element over the row's
+ * nonzeros and then k.  Needs no workspace; runs on `stream` (NULL = legacy
+ * default) asynchronously. */
+slnr_status slnr_spmm_gemm_original(const slnr_csr *B, const float *C, int32_t K, const float *D, int32_t L,
+                                    float *A, void *stream);
 
 /* ---- per-launch timing (instrumentation) --------------------------------
  * With timing enabled, each call on the calling thread records a CUDA event on

@@ -64,6 +64,7 @@ SIGNATURES = {
     "slnr_mttkrp_gemm_workspace": ([_CSF, _I32, _I32, _OPT, _SZ], ctypes.c_int),
     "slnr_spmmh_gemm_workspace": ([_CSR, _I32, _I32, _OPT, _SZ], ctypes.c_int),
     "slnr_spmm_gemm": ([_CSR, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
+    "slnr_spmm_gemm_original": ([_CSR, _P, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "slnr_sddmm_spmm": ([_CSR, _P, _P, _I32, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_mttkrp": ([_CSF, _P, _P, _I32, _P, _OPT], ctypes.c_int),
     "slnr_spttm_ttm": ([_CSF, _P, _I32, _P, _I32, _P, _P, _P, _P, _P, _OPT], ctypes.c_int),
@@ -347,6 +348,21 @@ def spmm_gemm(B: DeviceCSR, C, D, out=None, variant="fused", allow_tf32=True, va
     n = _query("slnr_spmm_gemm_workspace", ctypes.byref(bs), K, L, ctypes.byref(o))
     _keep = _attach_ws(o, n, workspace)
     _check(slnr_spmm_gemm(bs, C.data_ptr(), K, D.data_ptr(), L, out.data_ptr(), o), "slnr_spmm_gemm")
+    return out
+
+
+def spmm_gemm_original(B: DeviceCSR, C, D, out=None, stream=None):
+    """<SpMM,GEMM> as the perfect loop nest i, j, k, l (the comparator of
+    Sec. 6.3's case study; slnr_spmm_gemm_original)."""
+    torch = _torch()
+    C, D = _dense(C, "C"), _dense(D, "D")
+    K, L = C.shape[1], D.shape[1]
+    if out is None:
+        out = torch.empty((B.nrows, L), dtype=torch.float32, device=C.device)
+    bs = B.c_struct()
+    s = ctypes.c_void_p((stream or torch.cuda.current_stream()).cuda_stream)
+    _check(lib().slnr_spmm_gemm_original(ctypes.byref(bs), C.data_ptr(), K, D.data_ptr(), L, out.data_ptr(), s),
+           "slnr_spmm_gemm_original")
     return out
 
 

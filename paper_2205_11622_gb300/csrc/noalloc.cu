@@ -12,8 +12,7 @@
 // The host code must not use the array's name as a device pointer (in host
 // code it names a host-side stand-in), so the first call on each device looks
 // up the array's device address with cudaGetSymbolAddress, with that device
-// current, and caches it.  The first call on a device should therefore be
-// made before any stream capture begins.  The cache outlives a device reset
+// current, and caches it.  The cache outlives a device reset
 // (cudaDeviceReset), after which the address is stale: a process that
 // resets a device must not call this entry point on it again.  Every call shares the one array,
 // which keeps the last call's contents: the call clears the part that must

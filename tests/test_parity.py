@@ -299,3 +299,16 @@ def test_fused_call_routing(slnr, orc, op, size):
     assert on_tc == (size == "large"), names
     # every phase launches at least one kernel; none launches more than two
     assert len(names) <= launches <= 2 * len(names), (names, launches)
+
+
+@pytest.mark.parametrize("K,L", [(16, 16), (64, 128), (100, 36), (32, 260)])
+def test_spmm_gemm_original(slnr, orc, K, L):
+    # the perfect loop nest (the case study's comparator): the same A as the
+    # oracle; rows of 12 nonzeros keep each output's fp32 chain (12 K terms)
+    # within the fp32 tolerance; L = 260 leaves a ragged third column block
+    w = wl.spmm_gemm_uniform(0x51A4 + 3 * K + L, 300, 500, 12, K, L, name=f"original_{K}_{L}")
+    B, dense = P.to_device(w)
+    out = slnr.spmm_gemm_original(B, dense["C"], dense["D"])
+    torch.cuda.synchronize()
+    ref, ref_abs = orc.run(w)
+    assert P.rel_err(out.cpu().numpy(), ref, ref_abs) <= P.TOL_FP32

@@ -135,3 +135,9 @@ def test_widths_outside_the_contract_are_rejected():
     for K, L, want in ((6, 8, 5), (8, 1028, 5), (1024, 1024, 0), (0, 8, 2), (100, 12, 0)):
         st = lib.slnr_spmm_gemm_workspace(ctypes.byref(B), K, L, ctypes.byref(o), ctypes.byref(n))
         assert st == want, (K, L, st, m.last_error())
+        if want != 0:  # the perfect-loop-nest comparator checks its widths the same way, before any launch
+            st = lib.slnr_spmm_gemm_original(ctypes.byref(B), ctypes.c_void_p(0x1000), K, ctypes.c_void_p(0x2000), L,
+                                             ctypes.c_void_p(0x3000), None)
+            assert st == want, (K, L, st, m.last_error())
+    assert lib.slnr_spmm_gemm_original(ctypes.byref(B), None, 8, ctypes.c_void_p(0x2000), 8,
+                                       ctypes.c_void_p(0x3000), None) == 1
