@@ -1,8 +1,9 @@
-"""bench.py's useful-flop counts (the metric's numerator) against a scalar
-recount over the sparse structure, on every small workload and on CSF tensors
-with slices that hold no fibers.  The per-unit costs are the fused schedule's
-(Sec. 6.2): a dense row product per non-empty row or slice, a vector update per
-nonzero and per fiber."""
+"""bench.py's useful-flop counts (the metric's numerator) and byte counts (the
+roofline's numerators: referenced rows, every row, gathered rows) against
+scalar recounts over the sparse structure, on every small workload and on CSF
+tensors with slices that hold no fibers.  The per-unit costs are the fused
+schedule's (Sec. 6.2): a dense row product per non-empty row or slice, a vector
+update per nonzero and per fiber."""
 import numpy as np
 import pytest
 
@@ -71,3 +72,76 @@ def test_mttkrp_counts_with_fiberless_slices(op):
     per_row = bench.row_flops(w)
     assert per_row[2] == (2 * 8 * 4 if op == "mttkrp_gemm" else 0)  # a slice without fibers
     assert per_row[1] == 0 and per_row[4] == 0                       # rows without a slice
+
+
+def scalar_bytes(w, referenced_only=True):
+    """Bytes an ideal evaluation moves, recounted from the structure: index and
+    value arrays once, each dense row read once (only the rows a nonzero, a
+    non-empty row or a fiber refers to, with referenced_only), every output
+    element once."""
+    d, B = w.dims, w.B
+    dense = lambda name: w.dense[name] if name in w.dense else None
+    if w.op in ("spmm_gemm", "sddmm_spmm", "sddmm_spmm_gemm", "spmmh_gemm"):
+        cols = {int(c) for c in B.crd}
+        rows = [i for i in range(B.nrows) if B.pos[i + 1] > B.pos[i]]
+        total = 4 * (B.nrows + 1) + 8 * len(B.crd)
+        if w.op == "spmm_gemm":
+            K, L = d["K"], d["L"]
+            reads = (len(cols) if referenced_only else B.ncols) * 4 * K + 4 * K * L
+            return total + reads + 4 * B.nrows * L
+        if w.op == "sddmm_spmm":
+            K, L = d["K"], d["L"]
+            c_rows = len(rows) if referenced_only else B.nrows
+            return total + 4 * L * c_rows + (len(cols) if referenced_only else B.ncols) * 4 * (L + K) + 4 * B.nrows * K
+        if w.op == "sddmm_spmm_gemm":
+            K, L, M = d["K"], d["L"], d["M"]
+            c_rows = len(rows) if referenced_only else B.nrows
+            return (total + 4 * K * c_rows + (len(cols) if referenced_only else B.ncols) * 4 * (K + L) + 4 * L * M
+                    + 4 * B.nrows * M)
+        J, L = d["J"], d["L"]
+        return total + (len(cols) if referenced_only else B.ncols) * 8 * J + 4 * J * L + 4 * B.nrows * L
+    ns, nf, nnz = len(B.crd1), len(B.crd2), len(B.crd3)
+    structure = 8 + 4 * ns + 4 * (ns + 1) + 4 * nf + 4 * (nf + 1) + 8 * nnz
+    if w.op == "spttm_ttm":
+        L, M = d["L"], d["M"]
+        ks = len({int(k) for k in B.crd3}) if referenced_only else B.dims[2]
+        out_index = 8 + 4 * ns + 4 * (ns + 1) + 4 * nf
+        return structure + 4 * L * ks + 4 * L * M + 4 * nf * M + out_index
+    L = d["L"]
+    js = len({int(j) for j in B.crd2}) if referenced_only else B.dims[1]
+    ks = len({int(k) for k in B.crd3}) if referenced_only else B.dims[2]
+    if w.op == "mttkrp_gemm":
+        return structure + 4 * L * (js + ks) + 4 * L * d["M"] + 4 * B.dims[0] * d["M"]
+    return structure + 4 * L * (js + ks) + 4 * B.dims[0] * L
+
+
+def scalar_gather_bytes(w):
+    """Whole rows the fused producers read: one per nonzero (two for the
+    Hadamard and sampled rows), plus one C row per fiber for MTTKRP."""
+    d, B = w.dims, w.B
+    per = {"spmm_gemm": 4 * d.get("K", 0), "spttm_ttm": 4 * d.get("L", 0), "spmmh_gemm": 8 * d.get("J", 0),
+           "sddmm_spmm": 4 * (d.get("L", 0) + d.get("K", 0)), "sddmm_spmm_gemm": 4 * (d.get("K", 0) + d.get("L", 0)),
+           "mttkrp": 4 * d.get("L", 0), "mttkrp_gemm": 4 * d.get("L", 0)}[w.op]
+    total = 0
+    nnz = len(B.crd) if w.op in ("spmm_gemm", "sddmm_spmm", "sddmm_spmm_gemm", "spmmh_gemm") else len(B.crd3)
+    for _ in range(nnz):
+        total += per
+    if w.op in ("mttkrp", "mttkrp_gemm"):
+        total += 4 * d["L"] * len(B.crd2)
+    return total
+
+
+@pytest.mark.parametrize("kind,i", CASES)
+def test_byte_counts_match_a_recount(kind, i):
+    w = wl.small(i) if kind == "small" else wl.next_small(i)
+    assert bench.min_bytes(w) == scalar_bytes(w, referenced_only=True)
+    assert bench.gather_bytes(w) == scalar_gather_bytes(w)
+    assert bench.min_bytes_all_rows(w) == scalar_bytes(w, referenced_only=False)
+    assert bench.min_bytes_all_rows(w) >= bench.min_bytes(w)
+
+
+@pytest.mark.parametrize("width,want", [(4, 4), (12, 8), (32, 32), (100, 64), (128, 128), (512, 128), (1024, 128)])
+def test_gather_row_width_is_a_power_of_two_up_to_128(width, want):
+    B = wl.CSR(2, 2, np.asarray([0, 1, 1], np.int32), np.asarray([1], np.int32), np.ones(1, np.float32))
+    w = wl.Workload("w", "spmm_gemm", B, {}, {"K": width, "L": 8})
+    assert bench.gather_row_width(w) == want
