@@ -5,14 +5,15 @@
  * The library evaluates the four benchmark expressions of "SparseLNR:
  * Accelerating Sparse Tensor Computations Using Loop Nest Restructuring"
  * (Dias, Sundararajah, Saumya, Kulkarni; ICS'22, arXiv 2205.11622), Sec. 6.2,
- * with the schedule that the paper's "loop fusion after distribution"
+ * and three further expressions of the same section, with the schedule that the paper's "loop fusion after distribution"
  * (Sec. 4.2, Algorithm 1) derives: the outer sparse loop (CSR row, or CSF
  * slice / fiber) is shared by the producer and the consumer, the producer
  * fills a small temporary (a scalar or a vector) and the consumer uses it at
  * once, so the intermediate tensor is never written to memory.  Each entry
  * point also has an UNFUSED variant that materialises the intermediate in the
  * caller's workspace and runs producer and consumer as separate kernels (the
- * paper's "TACO Separate" baseline, Sec. 6).
+ * paper's "TACO Separate" baseline, Sec. 6); slnr_spmm_gemm_original runs
+ * <SpMM,GEMM> as the perfect loop nest (its "TACO Original").
  *
  * Conventions shared by every entry point
  *  - Every array argument (sparse structure, dense operands, outputs,
